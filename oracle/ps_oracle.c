@@ -1,0 +1,276 @@
+/*
+ * ps_oracle.c -- plain fp64 CPU reference for batched decode-phase attention
+ * over a paged KV cache with grouped-query heads.
+ *
+ * TEST INFRASTRUCTURE ONLY.  This file is the oracle that the CUDA path is
+ * checked against.  Only the test suite, the smoke check in
+ * __graft_entry__.py and the CPU-baseline leg of bench.py may load it.  It
+ * shares no code, header, table or helper with the CUDA library, and it never
+ * reads anything the CUDA library produced.
+ *
+ * What is computed (PowerSlider, Sec. 2.2: a decode step emits one new token
+ * per sequence and attends over every cached token of that sequence; the KV
+ * cache is the dominant byte stream, App. B.2 Eq. (bytes-layer), term 2BSd):
+ *
+ *   for each sequence s and query head h, with g = Hq / Hkv and KV head
+ *   j = h / g (contiguous grouping),
+ *
+ *     x_t  = scale * sum_d q[s][h][d] * K_s[t][d],        t = 0 .. L_s - 1
+ *     o[s][h][:] = sum_t exp(x_t - max_u x_u) V_s[t][:] / sum_t exp(x_t - max_u x_u)
+ *
+ *   where the logical token t of sequence s lives in physical block
+ *   b = block_table[s][t / bs], slot t % bs, and
+ *     K_s[t][:] = k_cache[b][j][t % bs][:]   (layout [num_blocks][Hkv][bs][d])
+ *     V_s[t][:] = v_cache[b][j][t % bs][:].
+ *   L_s = 0 gives an all-zero output row.
+ *
+ * Every input element is a bfloat16 bit pattern; it is widened exactly to
+ * double, and all arithmetic is double precision with libm exp().  Nothing
+ * is blocked, fused or reordered: each (s, h) row is a direct transcription
+ * of the definition above.
+ *
+ * ps_oracle_decode_attention_split() computes the same quantity by cutting
+ * each sequence's context into fixed chunks, keeping per chunk the running
+ * maximum m_c, the sum l_c = sum exp(x - m_c) and the weighted value sum
+ * acc_c, and merging the chunks with the log-sum-exp rule
+ *   o = sum_c exp(m_c - M) acc_c / sum_c exp(m_c - M) l_c,  M = max_c m_c.
+ * It exists so that the split-invariance of the definition can be pinned in
+ * the tests; it is not a different method.
+ *
+ * Pins (tests/test_oracle_pins.py): brute-force dense attention on logical
+ * arrays, closed forms (single token, constant V, zero query, equal keys),
+ * invariance to physical block relabelling, invariance to chunking,
+ * GQA == MHA with repeated KV heads, and torch's fp64 scaled-dot-product
+ * attention on tiny dense shapes.
+ *
+ * Error codes: 0 ok; -1 invalid argument; -2 a block id outside
+ * [0, num_blocks) is referenced; -3 a sequence length exceeds
+ * max_blocks_per_seq * block_size; -4 out of host memory.
+ */
+#include <math.h>
+#include <pthread.h>
+#include <stdatomic.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+static double bf16_bits_to_double(uint16_t bits)
+{
+    uint32_t u = ((uint32_t)bits) << 16;
+    float f;
+    memcpy(&f, &u, sizeof f);
+    return (double)f;
+}
+
+typedef struct {
+    const uint16_t *q;
+    const uint16_t *k_cache;
+    const uint16_t *v_cache;
+    const int32_t *block_table;
+    const int32_t *seq_lens;
+    int num_seqs, num_q_heads, num_kv_heads, head_dim, block_size;
+    int max_blocks_per_seq;
+    long long num_blocks;
+    double scale;
+    int chunk_tokens; /* 0: no chunking */
+    double *out;
+    atomic_int next_row;
+    atomic_int status;
+} job_t;
+
+/* Address of the first element of token t of sequence s, KV head j. */
+static const uint16_t *token_row(const job_t *jb, const uint16_t *cache, int s, int j, int t, int *err)
+{
+    int32_t b = jb->block_table[(size_t)s * jb->max_blocks_per_seq + t / jb->block_size];
+    if (b < 0 || (long long)b >= jb->num_blocks) {
+        *err = -2;
+        return NULL;
+    }
+    size_t page = (size_t)b * jb->num_kv_heads + (size_t)j;
+    return cache + (page * jb->block_size + (size_t)(t % jb->block_size)) * jb->head_dim;
+}
+
+/* One output row by the plain definition. */
+static int row_plain(job_t *jb, int s, int h, double *logits)
+{
+    const int d = jb->head_dim;
+    const int g = jb->num_q_heads / jb->num_kv_heads;
+    const int j = h / g;
+    const int L = jb->seq_lens[s];
+    const uint16_t *qv = jb->q + ((size_t)s * jb->num_q_heads + h) * d;
+    double *o = jb->out + ((size_t)s * jb->num_q_heads + h) * d;
+    int err = 0;
+
+    for (int i = 0; i < d; ++i) o[i] = 0.0;
+    if (L == 0) return 0;
+
+    double m = -INFINITY;
+    for (int t = 0; t < L; ++t) {
+        const uint16_t *kr = token_row(jb, jb->k_cache, s, j, t, &err);
+        if (err) return err;
+        double dot = 0.0;
+        for (int i = 0; i < d; ++i) dot += bf16_bits_to_double(qv[i]) * bf16_bits_to_double(kr[i]);
+        logits[t] = jb->scale * dot;
+        if (logits[t] > m) m = logits[t];
+    }
+    double z = 0.0;
+    for (int t = 0; t < L; ++t) {
+        double w = exp(logits[t] - m);
+        z += w;
+        const uint16_t *vr = token_row(jb, jb->v_cache, s, j, t, &err);
+        if (err) return err;
+        for (int i = 0; i < d; ++i) o[i] += w * bf16_bits_to_double(vr[i]);
+    }
+    for (int i = 0; i < d; ++i) o[i] /= z;
+    return 0;
+}
+
+/* The same row through per-chunk (m, l, acc) states merged by log-sum-exp. */
+static int row_split(job_t *jb, int s, int h, double *logits, double *acc_all, double *m_all, double *l_all)
+{
+    const int d = jb->head_dim;
+    const int g = jb->num_q_heads / jb->num_kv_heads;
+    const int j = h / g;
+    const int L = jb->seq_lens[s];
+    const int C = jb->chunk_tokens;
+    const uint16_t *qv = jb->q + ((size_t)s * jb->num_q_heads + h) * d;
+    double *o = jb->out + ((size_t)s * jb->num_q_heads + h) * d;
+    int err = 0;
+
+    for (int i = 0; i < d; ++i) o[i] = 0.0;
+    if (L == 0) return 0;
+
+    const int nchunks = (L + C - 1) / C;
+    for (int c = 0; c < nchunks; ++c) {
+        const int t0 = c * C;
+        const int t1 = (t0 + C < L) ? t0 + C : L;
+        double *acc = acc_all + (size_t)c * d;
+        double m = -INFINITY;
+        for (int t = t0; t < t1; ++t) {
+            const uint16_t *kr = token_row(jb, jb->k_cache, s, j, t, &err);
+            if (err) return err;
+            double dot = 0.0;
+            for (int i = 0; i < d; ++i) dot += bf16_bits_to_double(qv[i]) * bf16_bits_to_double(kr[i]);
+            logits[t] = jb->scale * dot;
+            if (logits[t] > m) m = logits[t];
+        }
+        double l = 0.0;
+        for (int i = 0; i < d; ++i) acc[i] = 0.0;
+        for (int t = t0; t < t1; ++t) {
+            double w = exp(logits[t] - m);
+            l += w;
+            const uint16_t *vr = token_row(jb, jb->v_cache, s, j, t, &err);
+            if (err) return err;
+            for (int i = 0; i < d; ++i) acc[i] += w * bf16_bits_to_double(vr[i]);
+        }
+        m_all[c] = m;
+        l_all[c] = l;
+    }
+    double M = -INFINITY;
+    for (int c = 0; c < nchunks; ++c)
+        if (m_all[c] > M) M = m_all[c];
+    double z = 0.0;
+    for (int c = 0; c < nchunks; ++c) {
+        double w = exp(m_all[c] - M);
+        z += w * l_all[c];
+        for (int i = 0; i < d; ++i) o[i] += w * acc_all[(size_t)c * d + i];
+    }
+    for (int i = 0; i < d; ++i) o[i] /= z;
+    return 0;
+}
+
+static void *worker(void *arg)
+{
+    job_t *jb = (job_t *)arg;
+    int maxL = 0;
+    for (int s = 0; s < jb->num_seqs; ++s)
+        if (jb->seq_lens[s] > maxL) maxL = jb->seq_lens[s];
+    double *logits = (double *)malloc(sizeof(double) * (size_t)(maxL > 0 ? maxL : 1));
+    double *acc = NULL, *ms = NULL, *ls = NULL;
+    if (jb->chunk_tokens > 0) {
+        size_t nc = (size_t)(maxL + jb->chunk_tokens - 1) / (size_t)jb->chunk_tokens + 1;
+        acc = (double *)malloc(sizeof(double) * nc * (size_t)jb->head_dim);
+        ms = (double *)malloc(sizeof(double) * nc);
+        ls = (double *)malloc(sizeof(double) * nc);
+    }
+    if (!logits || (jb->chunk_tokens > 0 && (!acc || !ms || !ls))) {
+        atomic_store(&jb->status, -4);
+        free(logits); free(acc); free(ms); free(ls);
+        return NULL;
+    }
+    const int rows = jb->num_seqs * jb->num_q_heads;
+    for (;;) {
+        int r = atomic_fetch_add(&jb->next_row, 1);
+        if (r >= rows || atomic_load(&jb->status) != 0) break;
+        int s = r / jb->num_q_heads, h = r % jb->num_q_heads;
+        int e = jb->chunk_tokens > 0 ? row_split(jb, s, h, logits, acc, ms, ls) : row_plain(jb, s, h, logits);
+        if (e) {
+            int zero = 0;
+            atomic_compare_exchange_strong(&jb->status, &zero, e);
+            break;
+        }
+    }
+    free(logits); free(acc); free(ms); free(ls);
+    return NULL;
+}
+
+static int run(job_t *jb, int num_threads)
+{
+    if (!jb->q || !jb->k_cache || !jb->v_cache || !jb->block_table || !jb->seq_lens || !jb->out) return -1;
+    if (jb->num_seqs < 0 || jb->num_q_heads <= 0 || jb->num_kv_heads <= 0 || jb->head_dim <= 0 ||
+        jb->block_size <= 0 || jb->max_blocks_per_seq < 0 || jb->num_blocks < 0 ||
+        jb->num_q_heads % jb->num_kv_heads != 0 || jb->chunk_tokens < 0)
+        return -1;
+    for (int s = 0; s < jb->num_seqs; ++s) {
+        if (jb->seq_lens[s] < 0) return -1;
+        if ((long long)jb->seq_lens[s] > (long long)jb->max_blocks_per_seq * jb->block_size) return -3;
+    }
+    atomic_init(&jb->next_row, 0);
+    atomic_init(&jb->status, 0);
+    if (num_threads < 1) num_threads = 1;
+    if (num_threads > 1024) num_threads = 1024;
+    pthread_t *tids = (pthread_t *)malloc(sizeof(pthread_t) * (size_t)num_threads);
+    if (!tids) return -4;
+    int started = 0;
+    for (int i = 0; i < num_threads; ++i) {
+        if (pthread_create(&tids[i], NULL, worker, jb) != 0) break;
+        ++started;
+    }
+    if (started == 0) worker(jb);
+    for (int i = 0; i < started; ++i) pthread_join(tids[i], NULL);
+    free(tids);
+    return atomic_load(&jb->status);
+}
+
+int ps_oracle_decode_attention(const uint16_t *q, const uint16_t *k_cache, const uint16_t *v_cache,
+                               const int32_t *block_table, const int32_t *seq_lens, int num_seqs,
+                               int num_q_heads, int num_kv_heads, int head_dim, int block_size,
+                               int max_blocks_per_seq, long long num_blocks, double scale,
+                               int num_threads, double *out)
+{
+    job_t jb;
+    memset(&jb, 0, sizeof jb);
+    jb.q = q; jb.k_cache = k_cache; jb.v_cache = v_cache;
+    jb.block_table = block_table; jb.seq_lens = seq_lens;
+    jb.num_seqs = num_seqs; jb.num_q_heads = num_q_heads; jb.num_kv_heads = num_kv_heads;
+    jb.head_dim = head_dim; jb.block_size = block_size; jb.max_blocks_per_seq = max_blocks_per_seq;
+    jb.num_blocks = num_blocks; jb.scale = scale; jb.chunk_tokens = 0; jb.out = out;
+    return run(&jb, num_threads);
+}
+
+int ps_oracle_decode_attention_split(const uint16_t *q, const uint16_t *k_cache, const uint16_t *v_cache,
+                                     const int32_t *block_table, const int32_t *seq_lens, int num_seqs,
+                                     int num_q_heads, int num_kv_heads, int head_dim, int block_size,
+                                     int max_blocks_per_seq, long long num_blocks, double scale,
+                                     int chunk_tokens, int num_threads, double *out)
+{
+    if (chunk_tokens <= 0) return -1;
+    job_t jb;
+    memset(&jb, 0, sizeof jb);
+    jb.q = q; jb.k_cache = k_cache; jb.v_cache = v_cache;
+    jb.block_table = block_table; jb.seq_lens = seq_lens;
+    jb.num_seqs = num_seqs; jb.num_q_heads = num_q_heads; jb.num_kv_heads = num_kv_heads;
+    jb.head_dim = head_dim; jb.block_size = block_size; jb.max_blocks_per_seq = max_blocks_per_seq;
+    jb.num_blocks = num_blocks; jb.scale = scale; jb.chunk_tokens = chunk_tokens; jb.out = out;
+    return run(&jb, num_threads);
+}
