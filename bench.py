@@ -1,0 +1,424 @@
+#!/usr/bin/env python
+"""Benchmark of paged GQA decode attention on GB300.
+
+One step = one decode-attention call (split-KV partial kernel + log-sum-exp
+combine) over one batch of a named synthetic workload whose inputs are
+already resident in HBM.  L2 is flushed (a 2x-L2 write) before every timed
+step, outside the timed interval, and each step is timed with CUDA events
+on the launching stream.
+
+Prints one JSON line.  Default workload: the Llama-3-8B-shaped decode layer
+(64 sequences, 32/8 heads, block 16, contexts U[1024, 4096]).  --config
+picks another of the five workloads.  --impl reference times the fp64 CPU
+oracle on the host cores instead (bounded samples of the same workload).
+
+Multi-GPU (torchrun, one process per GPU): every rank runs its own batch of
+the workload (weak scaling, no collective on the data path); the value is
+the KV bytes of all ranks over the slowest rank's time.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "decode-attention KV-read GB/s & fraction of HBM peak; decode tokens/s (1 GB300)"
+FALLBACK_HBM_GBS = 6800.0
+PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "ps_decode_partial_kernel_llama3-8b-decode.md")
+KERNEL_SOURCE = os.path.join(ROOT, "paper_2608_21719_gb300", "csrc", "ps_decode_kernels.cu")
+CLOCK_QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+
+def parse_args(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=300)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--config", type=int, default=2, choices=[1, 2, 3, 4, 5])
+    ap.add_argument("--cpu-seconds", type=float, default=12.0,
+                    help="CPU time budget of the oracle baseline sample")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args(argv)
+
+
+# ----------------------------------------------------------------- helpers --
+
+def dist_env():
+    return (int(os.environ.get("RANK", "0")), int(os.environ.get("LOCAL_RANK", "0")),
+            int(os.environ.get("WORLD_SIZE", "1")))
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def profiled_traffic():
+    """Per-launch DRAM bytes of the partial kernel from the committed ncu
+    summary, or None when the kernel source changed since it was taken."""
+    try:
+        text = open(PROFILE_SUMMARY).read()
+        src_hash = hashlib.sha256(open(KERNEL_SOURCE, "rb").read()).hexdigest()
+    except OSError:
+        return None
+    vals = {}
+    for line in text.splitlines():
+        line = line.strip().lstrip("-* ")
+        if ":" in line:
+            k, v = line.split(":", 1)
+            vals[k.strip().strip("`")] = v.strip().strip("`")
+    if vals.get("kernel_source_sha256") != src_hash:
+        return None
+    try:
+        return int(float(vals["traffic_bytes_per_launch"]))
+    except (KeyError, ValueError):
+        return None
+
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons during the timed region."""
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(prefix="ps_clocks_", suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), "--query-gpu=" + CLOCK_QUERY, "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        time.sleep(0.15)
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        if self.proc is None or self.path is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        rows = []
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) >= 9:
+                rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"], "samples": 0}
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return None
+        sm = [num(r[1]) for r in rows if num(r[1]) is not None]
+        mx = [num(r[2]) for r in rows if num(r[2]) is not None]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower() == "active"})
+        power = [num(r[3]) for r in rows if num(r[3]) is not None]
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows), "power_w_max": max(power) if power else None}
+
+
+def sample_for_oracle(wl, seq_idx, token_cap=None):
+    """Host copy of sequences ``seq_idx`` (optionally only their first
+    ``token_cap`` tokens) as a compact paged workload for the oracle."""
+    import numpy as np
+    import torch
+    from paper_2608_21719_gb300 import inputs
+    bs = wl.block_size
+    lens = wl.seq_lens[seq_idx].cpu().numpy().astype(np.int64)
+    if token_cap is not None:
+        lens = np.minimum(lens, token_cap)
+    bt = wl.block_table[seq_idx].cpu().numpy()
+    pages = [bt[i, :(int(L) + bs - 1) // bs] for i, L in enumerate(lens)]
+    flat = torch.from_numpy(np.concatenate(pages).astype(np.int64)).to(wl.k_cache.device)
+    k = wl.k_cache.index_select(0, flat).cpu()
+    v = wl.v_cache.index_select(0, flat).cpu()
+    nbt = np.full((len(seq_idx), max(1, max(len(p) for p in pages))), -1, dtype=np.int32)
+    pos = 0
+    for i, p in enumerate(pages):
+        nbt[i, :len(p)] = np.arange(pos, pos + len(p))
+        pos += len(p)
+    return inputs.Workload(cfg=None, q=wl.q[seq_idx].cpu(), k_cache=k, v_cache=v,
+                           block_table=torch.from_numpy(nbt), seq_lens=torch.from_numpy(lens.astype(np.int32)),
+                           scale=wl.scale)
+
+
+def time_oracle(sub, threads):
+    import oracle
+    from paper_2608_21719_gb300 import inputs, roofline
+    args = (inputs.bf16_bits(sub.q), inputs.bf16_bits(sub.k_cache), inputs.bf16_bits(sub.v_cache),
+            sub.block_table.numpy(), sub.seq_lens.numpy(), sub.num_kv_heads, sub.scale)
+    t0 = time.perf_counter()
+    oracle.decode_attention(*args, num_threads=threads)
+    dt = time.perf_counter() - t0
+    kv = roofline.algorithmic_bytes(sub.seq_lens.numpy(), sub.num_q_heads, sub.num_kv_heads, sub.head_dim,
+                                    sub.block_size)["kv"]
+    return dt, kv
+
+
+def choose_oracle_sample(wl, budget_s, threads):
+    """Sequences (in a fixed seeded order) and a token cap sized so that one
+    oracle run over them takes about ``budget_s`` seconds."""
+    import numpy as np
+    order = list(np.random.default_rng(12345).permutation(wl.num_seqs))
+    probe = sample_for_oracle(wl, order[:1], token_cap=512)
+    dt, kv = time_oracle(probe, threads)
+    rate = kv / max(dt, 1e-6)  # KV bytes per second of the oracle
+    want = rate * budget_s
+    lens = wl.seq_lens.cpu().numpy()
+    per_tok = 2 * wl.num_kv_heads * wl.head_dim * 2
+    chosen, acc = [], 0
+    for s in order:
+        b = int(lens[s]) * per_tok
+        if acc + b > want and chosen:
+            break
+        chosen.append(int(s))
+        acc += b
+    cap = None
+    if len(chosen) == 1 and acc > want:
+        cap = max(16, int(want // per_tok))
+    return chosen, cap
+
+
+# ------------------------------------------------------------- our arm ------
+
+def run_ours(args):
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    from paper_2608_21719_gb300 import inputs, ps_decode, roofline
+
+    rank, local_rank, world = dist_env()
+    if world > 1 and not dist.is_initialized():
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    cfg = inputs.CONFIGS[args.config]
+    wl = inputs.make_workload(cfg, device=dev, poison=False)
+    lens = wl.seq_lens.cpu().numpy()
+    alg = roofline.algorithmic_bytes(lens, wl.num_q_heads, wl.num_kv_heads, wl.head_dim, wl.block_size)
+    partial_bytes = alg["kv"] + alg["q"] + alg["block_table"] + alg["seq_lens"]
+
+    attn = ps_decode.DecodeAttention.for_workload(wl)
+    out = torch.empty_like(wl.q)
+    stream = torch.cuda.current_stream(dev)
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    flush = torch.empty(max(2 * l2, 64 << 20), dtype=torch.uint8, device=dev)
+
+    def step():
+        attn(wl.q, wl.k_cache, wl.v_cache, wl.block_table, wl.seq_lens, out=out, scale=wl.scale, stream=stream)
+
+    for _ in range(max(args.warmup, 3)):
+        flush.zero_()
+        step()
+    torch.cuda.synchronize(dev)
+    assert attn.device_status() == 0, "device status flags raised during warm-up"
+
+    K = args.steps
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)]
+    visible = [x.strip() for x in os.environ.get("CUDA_VISIBLE_DEVICES", "").split(",") if x.strip()]
+    gpu_index = visible[local_rank] if local_rank < len(visible) else str(local_rank)
+    n_launch0 = ps_decode.ps_decode_launch_count()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    with ClockSampler(gpu_index) as clk:
+        for k in range(K):
+            flush.zero_()
+            ps_decode.ps_decode_plan_set_timing_events(attn.plan, *ev[k])
+            step()
+        torch.cuda.synchronize(dev)
+    if world > 1:
+        dist.barrier()
+    launches = ps_decode.ps_decode_launch_count() - n_launch0
+    ps_decode.ps_decode_plan_set_timing_events(attn.plan, None, None, None)
+    step_ms = [e[0].elapsed_time(e[2]) for e in ev]
+    partial_ms = [e[0].elapsed_time(e[1]) for e in ev]
+    total_ms = sum(step_ms)
+    if world > 1:
+        t = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+
+    # End to end through the public API with host buffers: per step, copy the
+    # step's inputs (queries, block table, lengths) from pinned host memory,
+    # run the call, and read the output back.  The KV cache is the serving
+    # engine's resident state and stays in HBM.
+    q_h = wl.q.cpu().pin_memory()
+    bt_h = wl.block_table.cpu().pin_memory()
+    sl_h = wl.seq_lens.cpu().pin_memory()
+    out_h = torch.empty(out.shape, dtype=out.dtype).pin_memory()
+    q_d, bt_d, sl_d = torch.empty_like(wl.q), torch.empty_like(wl.block_table), torch.empty_like(wl.seq_lens)
+    e2e_steps = max(10, min(K, 100))
+    ee = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(e2e_steps)]
+    for i in range(e2e_steps + 3):
+        flush.zero_()
+        if i >= 3:
+            ee[i - 3][0].record(stream)
+        q_d.copy_(q_h, non_blocking=True)
+        bt_d.copy_(bt_h, non_blocking=True)
+        sl_d.copy_(sl_h, non_blocking=True)
+        attn(q_d, wl.k_cache, wl.v_cache, bt_d, sl_d, out=out, scale=wl.scale, stream=stream)
+        out_h.copy_(out, non_blocking=True)
+        if i >= 3:
+            ee[i - 3][1].record(stream)
+    torch.cuda.synchronize(dev)
+    e2e_ms = statistics.mean(a.elapsed_time(b) for a, b in ee)
+    h2d = q_h.numel() * 2 + bt_h.numel() * 4 + sl_h.numel() * 4
+    d2h = out_h.numel() * 2
+    assert torch.equal(out_h, out.cpu())
+
+    if rank != 0:
+        if world > 1:
+            dist.barrier()
+        return None
+
+    hbm_peak, peak_kind = measured_peaks()
+    ms_per_step = total_ms / K
+    value = alg["kv"] * world * K / (total_ms * 1e-3) / 1e9
+    mean_partial_ms = statistics.mean(partial_ms)
+    achieved = partial_bytes / (mean_partial_ms * 1e-3) / 1e9
+    line = {
+        "metric": METRIC,
+        "value": round(value, 2),
+        "unit": "GB/s",
+        "n_gpus": world,
+        "steps": K,
+        "warmup": args.warmup,
+        "ms_per_step": round(ms_per_step, 5),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic",
+        "config": {
+            "workload": cfg.name,
+            "num_seqs": wl.num_seqs, "num_q_heads": wl.num_q_heads, "num_kv_heads": wl.num_kv_heads,
+            "head_dim": wl.head_dim, "block_size": wl.block_size, "lengths": list(cfg.lengths),
+            "seed": cfg.seed, "total_tokens": int(lens.sum()), "kv_bytes": alg["kv"],
+            "pool_blocks": wl.num_blocks,
+            "l2": "flushed before every step (write of %d MB, outside the timed interval)" % (flush.numel() >> 20),
+            "parallelism": "replicas" if world == 1 else "dp%d (independent batches per GPU)" % world,
+        },
+        "frac_of_hbm_peak": round(alg["total"] / (ms_per_step * 1e-3) / 1e9 / hbm_peak, 4),
+        "decode_tokens_per_s": round(wl.num_seqs * world * K / (total_ms * 1e-3), 1),
+        "kernel_ms": {"partial_mean": round(mean_partial_ms, 5),
+                      "combine_mean": round(statistics.mean(e[1].elapsed_time(e[2]) for e in ev), 5)},
+        "roofline": {
+            "kernel": "ps_decode_partial_kernel",
+            "bound": "hbm",
+            "achieved": round(achieved, 1),
+            "peak": hbm_peak,
+            "peak_kind": peak_kind + " (copy bandwidth, burst)",
+            "unit": "GB/s",
+            "frac": round(achieved / hbm_peak, 4),
+            "traffic": profiled_traffic(),
+            "algorithmic_bytes_per_launch": partial_bytes,
+        },
+        "e2e": {"value": round(alg["kv"] / (e2e_ms * 1e-3) / 1e9, 2), "unit": "GB/s",
+                "ms_per_step": round(e2e_ms, 5), "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": int(launches),
+        "clocks": clk.summary(),
+        "plan": attn.info(),
+    }
+    if not args.no_cpu_baseline:
+        threads = os.cpu_count() or 1
+        chosen, cap = choose_oracle_sample(wl, args.cpu_seconds, threads)
+        sub = sample_for_oracle(wl, chosen, token_cap=cap)
+        dt, kv = time_oracle(sub, threads)
+        line["cpu_baseline"] = {
+            "value": round(kv / dt / 1e9, 4), "unit": "GB/s", "cores": threads, "kind": "oracle",
+            "sample": "%d of %d sequences%s of this workload, fp64 oracle, %.1f s" % (
+                len(chosen), wl.num_seqs, "" if cap is None else " (first %d tokens)" % cap, dt),
+        }
+    attn.close()
+    if world > 1:
+        dist.barrier()
+    return line
+
+
+# ------------------------------------------------------- reference arm ------
+
+def run_reference(args):
+    """The oracle, as it stands, on the host cores: each step runs it over a
+    bounded sample of the workload sized so that the whole run stays within
+    a few minutes."""
+    import torch
+
+    from paper_2608_21719_gb300 import inputs
+
+    rank, _, world = dist_env()
+    if rank != 0:
+        return None
+    cfg = inputs.CONFIGS[args.config]
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    wl = inputs.make_workload(cfg, device=dev, poison=False) if dev == "cuda" or args.config == 1 else None
+    if wl is None:
+        return {"impl": "reference", "unavailable": "workload %d needs a GPU to generate its inputs" % args.config}
+    threads = os.cpu_count() or 1
+    budget = max(0.05, 150.0 / max(1, args.steps + args.warmup))
+    chosen, cap = choose_oracle_sample(wl, budget, threads)
+    sub = sample_for_oracle(wl, chosen, token_cap=cap)
+    for _ in range(args.warmup):
+        time_oracle(sub, threads)
+    t = 0.0
+    kv = 0
+    for _ in range(args.steps):
+        dt, b = time_oracle(sub, threads)
+        t += dt
+        kv += b
+    value = kv / t / 1e9
+    sample = "%d of %d sequences%s per step" % (len(chosen), wl.num_seqs,
+                                                "" if cap is None else " (first %d tokens)" % cap)
+    return {
+        "impl": "reference",
+        "metric": METRIC, "value": round(value, 4), "unit": "GB/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(t / args.steps * 1e3, 3), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": cfg.name, "num_seqs": cfg.num_seqs, "num_q_heads": cfg.num_q_heads,
+                   "num_kv_heads": cfg.num_kv_heads, "head_dim": cfg.head_dim, "block_size": cfg.block_size},
+        "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": threads, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def main(argv=None):
+    args = parse_args(argv)
+    line = run_reference(args) if args.impl == "reference" else run_ours(args)
+    if line is not None:
+        print(json.dumps(line), flush=True)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,191 @@
+/*
+ * ps_decode.h -- C ABI of the GB300 (sm_103a) paged decode-attention library.
+ *
+ * The library computes batched decode-phase attention for the thinking and
+ * answer tokens of reasoning LLM serving (PowerSlider, Sec. 2.2: decode emits
+ * one token per sequence per step and is bound by reading the KV cache; App.
+ * B.2 Eq. (bytes-layer) charges it 2BSd bytes of KV per layer).  Every query
+ * head h of sequence s attends over all L_s cached tokens of that sequence:
+ *
+ *   o[s][h] = sum_{t < L_s} softmax_t(scale * q[s][h] . K_s[t]) V_s[t]
+ *
+ * with grouped-query heads (g = num_q_heads / num_kv_heads query heads share
+ * KV head h / g) and a paged KV cache addressed through a block table.
+ *
+ * ---------------------------------------------------------------- layouts --
+ *  q           bf16  [num_seqs][num_q_heads][head_dim]              contiguous
+ *  k_cache     bf16  [num_blocks][num_kv_heads][block_size][head_dim] contiguous
+ *  v_cache     bf16  same layout as k_cache
+ *  block_table int32 [num_seqs][max_blocks_per_seq] row-major; token t of
+ *              sequence s is slot t % block_size of physical block
+ *              block_table[s][t / block_size].  Entries past the last block a
+ *              sequence uses are never read.
+ *  seq_lens    int32 [num_seqs]; number of cached tokens of each sequence,
+ *              the current token included.  0 is allowed (output row = 0).
+ *  out         bf16  [num_seqs][num_q_heads][head_dim]; fully overwritten,
+ *              round-to-nearest-even from fp32.
+ *
+ * ----------------------------------------------------------- conventions --
+ *  - Every tensor pointer is a DEVICE pointer owned by the caller; the library
+ *    never allocates or frees device memory.  q, k_cache and v_cache must be
+ *    16-byte aligned; block_table and seq_lens 4-byte aligned; out 2-byte
+ *    aligned.
+ *  - Calls are asynchronous and ordered on the given CUDA stream
+ *    (cudaStream_t passed as void*; NULL is the legacy default stream).
+ *  - Supported shapes: head_dim == 128; 1 <= num_q_heads / num_kv_heads <= 8;
+ *    block_size a multiple of 16 in [16, 256]; 1 <= num_seqs <= 4096.
+ *    Other shapes return PS_ERR_UNSUPPORTED.
+ *  - Device-side values are not validated on the host.  A seq_lens value
+ *    above max_blocks_per_seq * block_size is clamped to it, and a block id
+ *    outside [0, num_blocks) reads zeros; both set a flag readable with
+ *    ps_decode_plan_read_device_status().  Nothing faults.
+ *  - Split-KV workspace: the caller allocates ps_decode_plan_create()'s
+ *    workspace_bytes of device memory and hands it to the plan.  One
+ *    workspace must not be used by two calls that can run concurrently.
+ *  - A plan is not thread-safe: use it from one host thread at a time.
+ */
+#ifndef PS_DECODE_H
+#define PS_DECODE_H
+
+#include <stddef.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef int ps_status_t;
+
+#define PS_OK 0
+#define PS_ERR_INVALID_ARG (-1) /* null pointer, bad dimension, misalignment */
+#define PS_ERR_UNSUPPORTED (-2) /* valid but outside the shapes listed above */
+#define PS_ERR_NO_PLAN (-3)     /* no plan bound to the stream, or dims differ */
+#define PS_ERR_WORKSPACE (-4)   /* workspace missing or smaller than planned */
+#define PS_ERR_CUDA (-5)        /* a CUDA runtime/driver call failed */
+
+/* Flags of the device status word (ps_decode_plan_read_device_status). */
+#define PS_DEVICE_TIMEOUT 1u       /* an in-kernel wait ran out; output invalid */
+#define PS_DEVICE_BAD_BLOCK 2u     /* a block id outside [0, num_blocks) was read */
+#define PS_DEVICE_LEN_CLAMPED 4u   /* a seq_lens entry exceeded the block-table row */
+
+typedef struct ps_decode_plan ps_decode_plan_t; /* opaque, host-owned */
+
+/* Read-only description of a plan, for tests and measurement. */
+typedef struct ps_decode_plan_info {
+    int num_seqs, num_q_heads, num_kv_heads, head_dim, block_size;
+    int max_blocks_per_seq;
+    long long num_blocks;
+    int num_sms;               /* SMs the grid is sized for */
+    int grid_ctas;             /* CTAs of the split-KV partial kernel */
+    int workers_per_cta;       /* independent streaming warps per CTA */
+    int stages_per_worker;     /* 16-token K/V tiles in flight per warp */
+    int max_workers;           /* cap on the balanced partition's worker count */
+    int min_stages_per_worker; /* floor on a worker's share, in 16-token tiles */
+    size_t workspace_bytes;
+    size_t smem_bytes;         /* dynamic shared memory of the partial kernel */
+} ps_decode_plan_info_t;
+
+/*
+ * Plan a decode-attention shape.  The plan fixes the grid of the split-KV
+ * partial kernel (one CTA per SM) and sizes the workspace that carries the
+ * per-worker partial (max, sum, weighted-value) states to the log-sum-exp
+ * combine.  No device memory is allocated.
+ *
+ *   max_blocks_per_seq  row stride of block_table (entries)
+ *   num_blocks          physical blocks in k_cache / v_cache (TMA bounds)
+ *   plan                out: new plan; free with ps_decode_plan_destroy()
+ *   workspace_bytes     out: device bytes the caller must provide
+ *
+ * Queries the current CUDA device for its SM count.  Errors:
+ * PS_ERR_INVALID_ARG (null out-pointers, non-positive dims, num_q_heads not a
+ * multiple of num_kv_heads), PS_ERR_UNSUPPORTED (shape outside the supported
+ * set), PS_ERR_CUDA (no device).
+ */
+ps_status_t ps_decode_plan_create(int num_seqs, int num_q_heads, int num_kv_heads, int head_dim,
+                                  int block_size, int max_blocks_per_seq, long long num_blocks,
+                                  ps_decode_plan_t **plan, size_t *workspace_bytes);
+
+/*
+ * As ps_decode_plan_create(), with explicit knobs (0 = default for each):
+ *   num_sms                SM count to size the grid for (0: query the device;
+ *                          a positive value needs no GPU, e.g. for host tests)
+ *   max_workers            upper bound on the number of balanced workers the
+ *                          kernel splits the batch's KV stream into
+ *                          (1 = no split at all)
+ *   min_stages_per_worker  smallest share of a worker, in 16-token tiles
+ *                          (1 = split as finely as the workers allow)
+ */
+ps_status_t ps_decode_plan_create_ex(int num_seqs, int num_q_heads, int num_kv_heads, int head_dim,
+                                     int block_size, int max_blocks_per_seq, long long num_blocks,
+                                     int num_sms, int max_workers, int min_stages_per_worker,
+                                     ps_decode_plan_t **plan, size_t *workspace_bytes);
+
+/* Give the plan its caller-owned device workspace (>= workspace_bytes, 256-byte
+ * aligned).  The first call after this zeroes the workspace's status word on
+ * that call's stream.  Errors: PS_ERR_INVALID_ARG, PS_ERR_WORKSPACE. */
+ps_status_t ps_decode_plan_set_workspace(ps_decode_plan_t *plan, void *workspace, size_t bytes);
+
+/* Bind the plan to a stream so that ps_decode_attention() on that stream
+ * uses it (the 13-argument call has no block-table stride and no workspace
+ * of its own).  Binding NULL plan removes the stream's binding.  A stream has
+ * at most one plan; rebinding replaces it.  Errors: none besides
+ * PS_ERR_INVALID_ARG for a destroyed plan. */
+ps_status_t ps_decode_plan_bind(ps_decode_plan_t *plan, void *stream);
+
+/* Destroy a plan and drop every stream binding to it.  NULL is a no-op. */
+ps_status_t ps_decode_plan_destroy(ps_decode_plan_t *plan);
+
+/* Fill *info with the plan's shape and launch configuration. */
+ps_status_t ps_decode_plan_info(const ps_decode_plan_t *plan, ps_decode_plan_info_t *info);
+
+/*
+ * Decode attention with the plan bound to `stream` (ps_decode_plan_bind).
+ * Launches the split-KV partial kernel and the log-sum-exp combine kernel on
+ * `stream`.  scale is applied to q . k before the softmax (1/sqrt(head_dim)
+ * for standard attention; any finite value is accepted).
+ *
+ * Errors: PS_ERR_NO_PLAN when no plan is bound to `stream` or its
+ * (num_seqs, num_q_heads, num_kv_heads, head_dim, block_size) differ from the
+ * arguments; PS_ERR_WORKSPACE when the plan has no workspace;
+ * PS_ERR_INVALID_ARG for null/misaligned pointers or a non-finite scale;
+ * PS_ERR_CUDA when a launch fails.  Nothing is launched on error.
+ */
+ps_status_t ps_decode_attention(const void *q, const void *k_cache, const void *v_cache,
+                                const int *block_table, const int *seq_lens, void *out,
+                                int num_seqs, int num_q_heads, int num_kv_heads, int head_dim,
+                                int block_size, float scale, void *stream);
+
+/* The same computation with an explicit plan (no stream binding needed). */
+ps_status_t ps_decode_attention_planned(const ps_decode_plan_t *plan, const void *q,
+                                        const void *k_cache, const void *v_cache,
+                                        const int *block_table, const int *seq_lens, void *out,
+                                        float scale, void *stream);
+
+/*
+ * Measurement hook: when events are set (cudaEvent_t as void*, NULL to
+ * clear), every call records ev_start before the partial kernel, ev_mid
+ * between the partial and the combine kernel, and ev_end after the combine,
+ * on the call's stream.
+ */
+ps_status_t ps_decode_plan_set_timing_events(ps_decode_plan_t *plan, void *ev_start, void *ev_mid,
+                                             void *ev_end);
+
+/* Copy the device status word (PS_DEVICE_* flags raised by calls since the
+ * last read) to *flags, synchronising `stream`, then clear it.  Errors:
+ * PS_ERR_WORKSPACE (no workspace), PS_ERR_CUDA. */
+ps_status_t ps_decode_plan_read_device_status(ps_decode_plan_t *plan, void *stream,
+                                              unsigned int *flags);
+
+/* Number of kernels this library has launched in this process. */
+unsigned long long ps_decode_launch_count(void);
+
+/* Static description of a status code. */
+const char *ps_status_string(ps_status_t status);
+
+/* ABI version of this header (major * 100 + minor). */
+int ps_decode_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PS_DECODE_H */

@@ -1,0 +1,605 @@
+// ps_decode_kernels.cu -- sm_103a kernels for batched paged GQA decode attention.
+//
+// Two launches per call:
+//
+//  1. ps_decode_partial_kernel (persistent, one CTA per SM, 4 independent
+//     worker warps per CTA).  The KV work of the whole batch is laid out as
+//     one "tape" of 16-token tiles, ordered by sequence and then KV head:
+//     segment (s, j) holds ceil(L_s / 16) tiles.  Every CTA rebuilds the
+//     per-sequence prefix sums of that tape in shared memory, and worker w of
+//     W gets the contiguous range [floor(w N / W), floor((w+1) N / W)) of the
+//     N tiles.  The split is therefore balanced to one tile whatever the mix
+//     of short answer-phase and long thinking-phase contexts (PowerSlider
+//     Sec. 2.2, Sec. 3 Obs. 3), with no atomics and no host knowledge of the
+//     lengths.  A worker streams its tiles through a ring of shared-memory
+//     stages filled by TMA (cp.async.bulk.tensor, 128-byte swizzle) and
+//     completed on mbarriers, reading each (block, kv-head) page exactly
+//     once for all g query heads of the group.  Per tile it computes the
+//     scores S^T = K Q^T and the update O^T += V^T P^T on the tensor cores
+//     (mma.sync m16n8k16, bf16 in, fp32 accumulate: tokens fill M = 16, the
+//     g <= 8 heads of the group fill N = 8), with an online softmax whose
+//     running max and sum stay in fp32.  A piece of a segment that a worker
+//     covers completely is normalised and written as bf16 output; a piece cut
+//     by a worker boundary leaves (m, l, acc) in the workspace.
+//
+//  2. ps_decode_combine_kernel merges the pieces of every cut segment with
+//     the log-sum-exp rule o = sum_c 2^(m_c - M) acc_c / sum_c 2^(m_c - M) l_c
+//     (scores are kept in base 2 with log2(e) folded into the scale), and
+//     zero-fills the rows of empty sequences.
+//
+// No wait spins forever: every mbarrier wait gives up after ~2 s of
+// globaltimer, raises PS_DEVICE_TIMEOUT in the workspace status word, drains
+// the worker's outstanding copies with the same bound and returns.
+#include <cuda_bf16.h>
+
+#include "ps_internal.h"
+
+namespace ps {
+namespace {
+
+constexpr unsigned kFull = 0xffffffffu;
+constexpr unsigned long long kWaitLimitNs = 2000000000ull;
+constexpr unsigned kFlagTimeout = 1u, kFlagBadBlock = 2u, kFlagLenClamped = 4u;
+
+// ------------------------------------------------------------ PTX wrappers --
+
+__device__ __forceinline__ uint32_t smem_addr(const void *p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void fence_mbar_init() {
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void fence_proxy_async_smem() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+__device__ __forceinline__ unsigned long long global_ns() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+// Bounded wait for phase `parity` of an mbarrier; false after ~2 s.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+    for (int i = 0; i < 256; ++i)
+        if (mbar_try_wait(bar, parity)) return true;
+    const unsigned long long t0 = global_ns();
+    while (!mbar_try_wait(bar, parity))
+        if (global_ns() - t0 > kWaitLimitNs) return false;
+    return true;
+}
+
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *tm, int c0, int c1, int c2,
+                                            uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(tm)), "r"(c0), "r"(c1), "r"(c2), "r"(bar)
+        : "memory");
+}
+
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void *src, uint32_t bytes, uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+        "l"(src), "r"(bytes), "r"(bar)
+        : "memory");
+}
+
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(addr)
+                 : "memory");
+}
+
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(addr)
+                 : "memory");
+}
+
+__device__ __forceinline__ uint32_t movm_t(uint32_t x) {
+    uint32_t y;
+    asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(y) : "r"(x));
+    return y;
+}
+
+// D = A(16x16 bf16, row) * B(16x8 bf16, col) + D, fp32 accumulate.
+__device__ __forceinline__ void mma_bf16(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                         uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+        "{%0, %1, %2, %3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+__device__ __forceinline__ float ex2(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+// Pack two floats to bf16x2 (round to nearest even); `lo` lands in bits 0..15.
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+    uint32_t r;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+    return r;
+}
+
+__device__ __forceinline__ float bf16lo(uint32_t x) { return __uint_as_float(x << 16); }
+__device__ __forceinline__ float bf16hi(uint32_t x) { return __uint_as_float(x & 0xffff0000u); }
+
+__device__ __forceinline__ uint16_t f2bf(float x) { return __bfloat16_as_ushort(__float2bfloat16_rn(x)); }
+
+// Byte offset of element (token, dim) inside a [half][16][64] tile written by
+// TMA with 128-byte swizzle: the 16-byte chunk index within a 128-byte row is
+// XORed with the row index mod 8 (stage buffers are 1024-byte aligned).
+__device__ __forceinline__ uint32_t tile_off(int token, int dim) {
+    return (uint32_t)((dim >> 6) * kHalfBytes + token * 128 + ((((dim & 63) >> 3) ^ (token & 7)) << 4));
+}
+
+// --------------------------------------------------------- tape cursor ----
+
+struct Cursor {
+    int s, h, st, ns;  // sequence, kv head, tile within segment, tiles in segment
+};
+
+__device__ __forceinline__ int tiles_of(int len) { return (len + kTileTokens - 1) / kTileTokens; }
+
+__device__ __forceinline__ Cursor locate(const int *sP, const int *sL, int S, int Hkv, int x) {
+    int lo = 0, hi = S - 1;
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (sP[mid] <= x) lo = mid; else hi = mid - 1;
+    }
+    Cursor c;
+    c.s = lo;
+    c.ns = tiles_of(sL[lo]);
+    const int off = x - sP[lo];
+    c.h = off / c.ns;
+    c.st = off - c.h * c.ns;
+    (void)Hkv;
+    return c;
+}
+
+__device__ __forceinline__ void advance(Cursor &c, const int *sL, int S, int Hkv) {
+    if (++c.st < c.ns) return;
+    c.st = 0;
+    if (++c.h < Hkv) return;
+    c.h = 0;
+    do {
+        ++c.s;
+    } while (c.s < S && sL[c.s] == 0);
+    c.ns = c.s < S ? tiles_of(sL[c.s]) : 0;
+}
+
+// ------------------------------------------------------ partial kernel ----
+
+__global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
+    ps_decode_partial_kernel(const PartialParams p, const __grid_constant__ CUtensorMap tmK,
+                             const __grid_constant__ CUtensorMap tmV) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kWorkersPerCta * kWorkerBytes);
+    int *sP = reinterpret_cast<int *>(bars + kWorkersPerCta * kStages);  // [S + 1] tile prefix (x Hkv)
+    int *sL = sP + p.num_seqs + 1;                                        // [S] clamped lengths
+    __shared__ int warp_sums[kWorkersPerCta];
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int S = p.num_seqs, Hkv = p.num_kv_heads, g = p.group, bs = p.block_size;
+
+    // 1. Clamped lengths and the exclusive prefix of tiles x kv-heads.
+    {
+        const int nthr = blockDim.x;
+        const int per = (S + nthr - 1) / nthr;
+        const int lo = min(S, tid * per), hi = min(S, lo + per);
+        int sum = 0;
+        bool clamped = false;
+        for (int i = lo; i < hi; ++i) {
+            int L = p.seq_lens[i];
+            if (L > p.len_cap) { L = p.len_cap; clamped = true; }
+            if (L < 0) L = 0;
+            sL[i] = L;
+            sum += tiles_of(L) * Hkv;
+        }
+        if (clamped && blockIdx.x == 0) atomicOr(reinterpret_cast<unsigned *>(p.ws_header + kHdrStatus), kFlagLenClamped);
+        int incl = sum;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int v = __shfl_up_sync(kFull, incl, o);
+            if (lane >= o) incl += v;
+        }
+        if (lane == 31) warp_sums[warp] = incl;
+        __syncthreads();
+        int run = incl - sum;
+        for (int i = 0; i < warp; ++i) run += warp_sums[i];
+        for (int i = lo; i < hi; ++i) {
+            sP[i] = run;
+            run += tiles_of(sL[i]) * Hkv;
+        }
+        if (lo < hi && hi == S) sP[S] = run;
+        if (lane == 0)
+            for (int i = 0; i < kStages; ++i) mbar_init(smem_addr(&bars[warp * kStages + i]), 1);
+        fence_mbar_init();
+        __syncthreads();
+    }
+
+    const int N = sP[S];
+    long long W = (long long)gridDim.x * kWorkersPerCta;
+    if (p.max_workers > 0 && W > p.max_workers) W = p.max_workers;
+    {
+        const long long cap = (N + p.min_stages - 1) / p.min_stages;
+        if (W > cap) W = cap;
+    }
+    if (blockIdx.x == 0) {
+        for (int i = tid; i <= S; i += blockDim.x) p.ws_prefix[i] = sP[i];
+        if (tid == 0) {
+            p.ws_header[kHdrTotalStages] = N;
+            p.ws_header[kHdrWorkers] = (int)W;
+        }
+    }
+    // Worker ids interleave CTAs first so that a small W still spreads over SMs.
+    const int w = warp * gridDim.x + blockIdx.x;
+    if (N == 0 || w >= W) return;
+    const int begin = (int)((long long)w * N / W);
+    const int total = (int)((long long)(w + 1) * N / W) - begin;
+    if (total <= 0) return;
+
+    uint8_t *wbase = smem + warp * kWorkerBytes;
+    uint8_t *qslots = wbase + kStages * kStageBytes;
+    uint64_t *wbars = bars + warp * kStages;
+    const int mbps = p.max_blocks_per_seq;
+
+    // ---- issue side: TMA producer state (lane 0 issues, all lanes track) ----
+    Cursor ic = locate(sP, sL, S, Hkv, begin);
+    int issued = 0, pieces_issued = 0;
+    int win_s = -1, win_j0 = 0, win_v = -1;  // block-table window, one entry per lane
+    int pre_s = -1, pre_j0 = 0, pre_v = -1;  // prefetched next window
+
+    auto fetch_window = [&](int s, int j0) -> int {
+        const int j = j0 + lane;
+        const int np = (sL[s] + bs - 1) / bs;
+        return j < np ? __ldg(p.block_table + (size_t)s * mbps + j) : -1;
+    };
+    // Start loading the window the issue cursor will need after the current one.
+    auto prefetch_next = [&]() {
+        int ns_ = -1, nj0 = 0;
+        const int np = (sL[ic.s] + bs - 1) / bs;
+        if (win_j0 + 32 < np) {
+            ns_ = ic.s; nj0 = win_j0 + 32;
+        } else if (ic.h + 1 < Hkv) {
+            ns_ = ic.s; nj0 = 0;
+        } else {
+            int s2 = ic.s + 1;
+            while (s2 < S && sL[s2] == 0) ++s2;
+            if (s2 < S) { ns_ = s2; nj0 = 0; }
+        }
+        if (ns_ < 0 || (ns_ == win_s && nj0 == win_j0) || (ns_ == pre_s && nj0 == pre_j0)) return;
+        pre_s = ns_; pre_j0 = nj0;
+        pre_v = fetch_window(ns_, nj0);
+    };
+
+    auto issue_one = [&]() {
+        const int slot = issued % kStages;
+        const bool new_piece = issued == 0 || ic.st == 0;
+        const int tok = ic.st * kTileTokens;
+        const int j = tok / bs, tok0 = tok - j * bs, j0 = j & ~31;
+        if (win_s != ic.s || win_j0 != j0) {
+            if (pre_s == ic.s && pre_j0 == j0) {
+                win_v = pre_v; pre_s = -1;
+            } else {
+                win_v = fetch_window(ic.s, j0);
+            }
+            win_s = ic.s; win_j0 = j0;
+            prefetch_next();
+        } else if (new_piece) {
+            prefetch_next();
+        }
+        const int pb = __shfl_sync(kFull, win_v, j - j0);
+        if (lane == 0) {
+            int row = pb * Hkv + ic.h;
+            if (pb < 0 || (long long)pb >= p.num_blocks) {
+                row = -1;  // fully out of bounds: TMA fills zeros
+                atomicOr(reinterpret_cast<unsigned *>(p.ws_header + kHdrStatus), kFlagBadBlock);
+            }
+            const uint32_t bar = smem_addr(&wbars[slot]);
+            const uint32_t dst = smem_addr(wbase + slot * kStageBytes);
+            const uint32_t qbytes = new_piece ? (uint32_t)(g * kHeadDim * 2) : 0u;
+            fence_proxy_async_smem();
+            mbar_arrive_expect_tx(bar, kStageBytes + qbytes);
+            tma_load_3d(dst, &tmK, 0, tok0, row, bar);
+            tma_load_3d(dst + kHalfBytes, &tmK, 64, tok0, row, bar);
+            tma_load_3d(dst + kTileBytes, &tmV, 0, tok0, row, bar);
+            tma_load_3d(dst + kTileBytes + kHalfBytes, &tmV, 64, tok0, row, bar);
+            if (new_piece) {
+                const uint16_t *qsrc = p.q + ((size_t)ic.s * p.num_q_heads + (size_t)ic.h * g) * kHeadDim;
+                bulk_load(smem_addr(qslots + (pieces_issued % kQSlots) * kQSlotBytes), qsrc, qbytes, bar);
+            }
+        }
+        if (new_piece) ++pieces_issued;
+        ++issued;
+        if (issued < total) advance(ic, sL, S, Hkv);
+    };
+
+    // ---- consume side state ----
+    Cursor cc = locate(sP, sL, S, Hkv, begin);
+    int pieces_loaded = 0;
+    bool first_piece = true, piece_from_start = false;
+    uint32_t qf[16];
+    float acc[8][4];
+    float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
+
+    auto refill = [&](int consumed) {
+        while (issued < total && issued - consumed < kStages) {
+            const bool np_ = issued == 0 || ic.st == 0;
+            if (np_ && pieces_issued >= pieces_loaded + kQSlots) break;
+            issue_one();
+        }
+    };
+
+    refill(0);
+    const int h0 = 2 * (lane & 3), h1 = h0 + 1;
+    const int trow = lane >> 2;  // token row of this lane in the S^T fragment
+    int consumed = 0;
+    for (; consumed < total;) {
+        const int slot = consumed % kStages;
+        const bool arrived = mbar_wait(smem_addr(&wbars[slot]), (uint32_t)((consumed / kStages) & 1));
+        if (!__all_sync(kFull, arrived)) {
+            if (lane == 0) atomicOr(reinterpret_cast<unsigned *>(p.ws_header + kHdrStatus), kFlagTimeout);
+            // Drain this worker's outstanding copies (bounded) before leaving.
+            for (int k = consumed + 1; k < issued; ++k)
+                mbar_wait(smem_addr(&wbars[k % kStages]), (uint32_t)((k / kStages) & 1));
+            return;
+        }
+        const uint8_t *stage = wbase + slot * kStageBytes;
+        const uint32_t sK = smem_addr(stage), sV = sK + kTileBytes;
+        const bool piece_start = consumed == 0 || cc.st == 0;
+        const bool seg_last = cc.st == cc.ns - 1;
+        const bool piece_end = consumed == total - 1 || seg_last;
+
+        if (piece_start) {
+            const uint32_t qs = smem_addr(qslots + (pieces_loaded % kQSlots) * kQSlotBytes);
+#pragma unroll
+            for (int kp = 0; kp < 4; ++kp)
+                ldsm_x4(qs + (lane & 7) * (kHeadDim * 2) + (32 * kp + 8 * (lane >> 3)) * 2, qf[4 * kp], qf[4 * kp + 1],
+                        qf[4 * kp + 2], qf[4 * kp + 3]);
+            if ((lane >> 2) >= g) {
+#pragma unroll
+                for (int i = 0; i < 16; ++i) qf[i] = 0u;
+            }
+            ++pieces_loaded;
+            piece_from_start = cc.st == 0;
+            m0 = m1 = -INFINITY;
+            l0 = l1 = 0.f;
+#pragma unroll
+            for (int mt = 0; mt < 8; ++mt) acc[mt][0] = acc[mt][1] = acc[mt][2] = acc[mt][3] = 0.f;
+        }
+
+        // S^T (16 tokens x 8 heads) = K (16 x 128) . Q^T (128 x 8), two accumulation chains.
+        float sa[4] = {0.f, 0.f, 0.f, 0.f}, sb[4] = {0.f, 0.f, 0.f, 0.f};
+        {
+            const int tok = (lane & 7) + ((lane >> 3) & 1) * 8;
+            const int dsub = (lane >> 4) * 8;
+#pragma unroll
+            for (int kk = 0; kk < 8; ++kk) {
+                uint32_t a0, a1, a2, a3;
+                ldsm_x4(sK + tile_off(tok, kk * 16 + dsub), a0, a1, a2, a3);
+                if (kk & 1) mma_bf16(sb, a0, a1, a2, a3, qf[2 * kk], qf[2 * kk + 1]);
+                else mma_bf16(sa, a0, a1, a2, a3, qf[2 * kk], qf[2 * kk + 1]);
+            }
+        }
+        const int n_valid = seg_last ? sL[cc.s] - (cc.ns - 1) * kTileTokens : kTileTokens;
+        float x0 = (sa[0] + sb[0]) * p.scale_log2, x1 = (sa[1] + sb[1]) * p.scale_log2;
+        float x2 = (sa[2] + sb[2]) * p.scale_log2, x3 = (sa[3] + sb[3]) * p.scale_log2;
+        if (trow >= n_valid) x0 = x1 = -INFINITY;
+        if (trow + 8 >= n_valid) x2 = x3 = -INFINITY;
+        if (n_valid < kTileTokens) {
+            // Tail of the sequence: zero the V rows past the last token so that
+            // 0-weights never meet stale or NaN data in the P.V product.
+            const int rows = kTileTokens - n_valid;
+            uint8_t *vt = const_cast<uint8_t *>(stage) + kTileBytes;
+            for (int i = lane; i < rows * 16; i += 32) {
+                const int r = n_valid + (i >> 4), half = (i >> 3) & 1, c = i & 7;
+                *reinterpret_cast<uint4 *>(vt + half * kHalfBytes + r * 128 + c * 16) = make_uint4(0, 0, 0, 0);
+            }
+            // These generic-proxy writes must be ordered before the TMA that
+            // later refills this stage.
+            fence_proxy_async_smem();
+            __syncwarp();
+        }
+        float mx0 = fmaxf(x0, x2), mx1 = fmaxf(x1, x3);
+#pragma unroll
+        for (int o = 4; o < 32; o <<= 1) {
+            mx0 = fmaxf(mx0, __shfl_xor_sync(kFull, mx0, o));
+            mx1 = fmaxf(mx1, __shfl_xor_sync(kFull, mx1, o));
+        }
+        const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);  // finite: a tile has >= 1 valid token
+        const float al0 = ex2(m0 - mn0), al1 = ex2(m1 - mn1);
+        m0 = mn0;
+        m1 = mn1;
+        const uint32_t P01 = pack_bf16(ex2(x0 - mn0), ex2(x1 - mn1));  // token trow
+        const uint32_t P23 = pack_bf16(ex2(x2 - mn0), ex2(x3 - mn1));  // token trow + 8
+        l0 = l0 * al0 + bf16lo(P01) + bf16lo(P23);
+        l1 = l1 * al1 + bf16hi(P01) + bf16hi(P23);
+#pragma unroll
+        for (int mt = 0; mt < 8; ++mt) {
+            acc[mt][0] *= al0; acc[mt][1] *= al1; acc[mt][2] *= al0; acc[mt][3] *= al1;
+        }
+        // P^T fragments (k = token, n = head) by transposing the bf16 score tiles.
+        const uint32_t pb0 = movm_t(P01), pb1 = movm_t(P23);
+
+        // O^T (128 x 8) += V^T (128 x 16) . P^T (16 x 8)
+        {
+            const int j = lane >> 3;
+            const int tok = (lane & 7) + (j >> 1) * 8;
+            const int dsub = (j & 1) * 8;
+#pragma unroll
+            for (int mt = 0; mt < 8; ++mt) {
+                uint32_t a0, a1, a2, a3;
+                ldsm_x4_t(sV + tile_off(tok, mt * 16 + dsub), a0, a1, a2, a3);
+                mma_bf16(acc[mt], a0, a1, a2, a3, pb0, pb1);
+            }
+        }
+
+        if (piece_end) {
+            float L0 = l0, L1 = l1;
+#pragma unroll
+            for (int o = 4; o < 32; o <<= 1) {
+                L0 += __shfl_xor_sync(kFull, L0, o);
+                L1 += __shfl_xor_sync(kFull, L1, o);
+            }
+            const int drow = lane >> 2;
+            if (piece_from_start && seg_last) {
+                // The worker saw the whole segment: write the bf16 output rows.
+                uint16_t *o = p.out + ((size_t)cc.s * p.num_q_heads + (size_t)cc.h * g) * kHeadDim;
+                const float i0 = 1.f / L0, i1 = 1.f / L1;
+#pragma unroll
+                for (int mt = 0; mt < 8; ++mt) {
+                    const int d = mt * 16 + drow;
+                    if (h0 < g) {
+                        o[h0 * kHeadDim + d] = f2bf(acc[mt][0] * i0);
+                        o[h0 * kHeadDim + d + 8] = f2bf(acc[mt][2] * i0);
+                    }
+                    if (h1 < g) {
+                        o[h1 * kHeadDim + d] = f2bf(acc[mt][1] * i1);
+                        o[h1 * kHeadDim + d + 8] = f2bf(acc[mt][3] * i1);
+                    }
+                }
+            } else {
+                // Cut by a worker boundary: leave (m, l, acc) for the combine.
+                const size_t slotid = 2 * (size_t)w + (first_piece ? 0 : 1);
+                float *A = p.ws_acc + slotid * kSlotFloats;
+#pragma unroll
+                for (int mt = 0; mt < 8; ++mt) {
+                    const int d = mt * 16 + drow;
+                    A[h0 * kHeadDim + d] = acc[mt][0];
+                    A[h0 * kHeadDim + d + 8] = acc[mt][2];
+                    A[h1 * kHeadDim + d] = acc[mt][1];
+                    A[h1 * kHeadDim + d + 8] = acc[mt][3];
+                }
+                if (lane < 4) {
+                    float *ML = p.ws_ml + slotid * kSlotMl;
+                    ML[2 * h0] = m0; ML[2 * h0 + 1] = L0;
+                    ML[2 * h1] = m1; ML[2 * h1 + 1] = L1;
+                }
+            }
+            first_piece = false;
+        }
+        ++consumed;
+        if (consumed < total) advance(cc, sL, S, Hkv);
+        refill(consumed);
+    }
+}
+
+// ------------------------------------------------------ combine kernel ----
+
+__device__ __forceinline__ int worker_of(long long x, long long N, long long W) {
+    return (int)(((x + 1) * W - 1) / N);
+}
+
+constexpr int kCombineWarps = 8;
+
+__global__ void __launch_bounds__(kCombineWarps * 32) ps_decode_combine_kernel(const CombineParams p) {
+    const int s = blockIdx.x;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int g = p.group;
+    const long long N = p.ws_header[kHdrTotalStages];
+    const long long W = p.ws_header[kHdrWorkers];
+    const int P0 = p.ws_prefix[s], P1 = p.ws_prefix[s + 1];
+    const int ns = (P1 - P0) / p.num_kv_heads;
+    for (int h = warp; h < p.num_kv_heads; h += kCombineWarps) {
+        uint16_t *o = p.out + ((size_t)s * p.num_q_heads + (size_t)h * g) * kHeadDim;
+        if (ns == 0) {
+            for (int i = lane; i < g * kHeadDim; i += 32) o[i] = 0;
+            continue;
+        }
+        const long long a = P0 + (long long)h * ns, b = a + ns;
+        const int wf = worker_of(a, N, W), wl = worker_of(b - 1, N, W);
+        if (wf == wl) continue;  // the partial kernel wrote this segment
+        const long long Rf = (long long)wf * N / W;
+        auto slot_of = [&](int wk) -> size_t {
+            return (wk == wf && Rf != a) ? 2 * (size_t)wk + 1 : 2 * (size_t)wk;
+        };
+        for (int n = 0; n < g; ++n) {
+            float M = -INFINITY;
+            for (int wk = wf + lane; wk <= wl; wk += 32) M = fmaxf(M, p.ws_ml[slot_of(wk) * kSlotMl + 2 * n]);
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(kFull, M, off));
+            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+            float lsum = 0.f;
+            for (int w0 = wf; w0 <= wl; w0 += 32) {
+                const int wk = w0 + lane;
+                float e = 0.f;
+                if (wk <= wl) {
+                    const float *ml = p.ws_ml + slot_of(wk) * kSlotMl + 2 * n;
+                    e = ex2(ml[0] - M);
+                    lsum += e * ml[1];
+                }
+                const int cnt = min(32, wl - w0 + 1);
+                for (int i = 0; i < cnt; ++i) {
+                    const float ei = __shfl_sync(kFull, e, i);
+                    const float4 v = *reinterpret_cast<const float4 *>(p.ws_acc + slot_of(w0 + i) * kSlotFloats +
+                                                                       (size_t)n * kHeadDim + 4 * lane);
+                    acc.x += ei * v.x; acc.y += ei * v.y; acc.z += ei * v.z; acc.w += ei * v.w;
+                }
+            }
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1) lsum += __shfl_xor_sync(kFull, lsum, off);
+            const float inv = 1.f / lsum;
+            uint16_t *on = o + n * kHeadDim + 4 * lane;
+            on[0] = f2bf(acc.x * inv); on[1] = f2bf(acc.y * inv);
+            on[2] = f2bf(acc.z * inv); on[3] = f2bf(acc.w * inv);
+        }
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_partial(const PartialParams &p, const CUtensorMap &tmK, const CUtensorMap &tmV, int grid_ctas,
+                           size_t smem_bytes, cudaStream_t stream) {
+    static bool attr_done[64] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    if (!attr_done[dev]) {
+        e = cudaFuncSetAttribute(ps_decode_partial_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)partial_smem_bytes(kMaxSeqs));
+        if (e != cudaSuccess) return e;
+        attr_done[dev] = true;
+    }
+    ps_decode_partial_kernel<<<grid_ctas, kWorkersPerCta * 32, smem_bytes, stream>>>(p, tmK, tmV);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_combine(const CombineParams &p, cudaStream_t stream) {
+    ps_decode_combine_kernel<<<p.num_seqs, kCombineWarps * 32, 0, stream>>>(p);
+    return cudaGetLastError();
+}
+
+}  // namespace ps

@@ -134,6 +134,11 @@ class Workload:
     seq_lens: torch.Tensor     # [S] int32
     scale: float
 
+    def to(self, device) -> "Workload":
+        return Workload(cfg=self.cfg, q=self.q.to(device), k_cache=self.k_cache.to(device),
+                        v_cache=self.v_cache.to(device), block_table=self.block_table.to(device),
+                        seq_lens=self.seq_lens.to(device), scale=self.scale)
+
     @property
     def num_seqs(self) -> int:
         return self.q.shape[0]

@@ -1,0 +1,151 @@
+"""Host-side checks of the C ABI (no GPU needed).
+
+The library must load, export every function include/ps_decode.h declares,
+reject bad arguments before touching the device, and size plans and
+workspaces as documented.  No call here launches a kernel.
+"""
+import ctypes
+
+import pytest
+
+from paper_2608_21719_gb300 import build as _build
+
+_build.build()
+from paper_2608_21719_gb300 import ps_decode as psd  # noqa: E402
+
+
+def test_every_declared_symbol_is_exported():
+    names = psd.header_functions()
+    expected = {"ps_decode_plan_create", "ps_decode_plan_create_ex", "ps_decode_plan_set_workspace",
+                "ps_decode_plan_bind", "ps_decode_plan_destroy", "ps_decode_plan_info", "ps_decode_attention",
+                "ps_decode_attention_planned", "ps_decode_plan_set_timing_events",
+                "ps_decode_plan_read_device_status", "ps_decode_launch_count", "ps_status_string",
+                "ps_decode_abi_version"}
+    assert expected <= set(names)
+    lib = ctypes.CDLL(psd.LIB_PATH)
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def test_status_strings_and_version():
+    assert psd.ps_status_string(0) == "ok"
+    for s in (-1, -2, -3, -4, -5):
+        assert psd.ps_status_string(s) not in ("ok", "unknown status")
+    assert psd.ps_status_string(-99) == "unknown status"
+    assert psd.ps_decode_abi_version() == 100
+
+
+def _plan(**kw):
+    args = dict(num_seqs=64, num_q_heads=32, num_kv_heads=8, head_dim=128, block_size=16, max_blocks_per_seq=256,
+                num_blocks=12000, num_sms=152, max_workers=0, min_stages_per_worker=0)
+    args.update(kw)
+    return psd.ps_decode_plan_create_ex(**args)
+
+
+def test_plan_sizing_matches_layout():
+    plan, ws = _plan()
+    try:
+        info = psd.ps_decode_plan_info(plan)
+        assert info["grid_ctas"] == 152
+        assert info["workers_per_cta"] == 4
+        W = 152 * 4
+        assert info["max_workers"] == W
+        # header + prefix (S + 1 ints) + 2W partial slots of 8 heads x (128 acc + m, l) fp32
+        expect = 256 + 512 + 2 * W * 8 * 128 * 4 + 2 * W * 8 * 2 * 4
+        assert ws == info["workspace_bytes"]
+        assert expect <= ws <= expect + 3 * 256
+        assert info["smem_bytes"] <= 227 * 1024
+    finally:
+        psd.ps_decode_plan_destroy(plan)
+
+
+def test_max_seqs_plan_fits_shared_memory():
+    plan, ws = _plan(num_seqs=4096)
+    try:
+        assert psd.ps_decode_plan_info(plan)["smem_bytes"] <= 227 * 1024
+    finally:
+        psd.ps_decode_plan_destroy(plan)
+
+
+@pytest.mark.parametrize("kw,status", [
+    (dict(num_seqs=0), psd.PS_ERR_INVALID_ARG),
+    (dict(num_q_heads=30, num_kv_heads=8), psd.PS_ERR_INVALID_ARG),
+    (dict(head_dim=64), psd.PS_ERR_UNSUPPORTED),
+    (dict(num_q_heads=128, num_kv_heads=8), psd.PS_ERR_UNSUPPORTED),
+    (dict(block_size=8), psd.PS_ERR_UNSUPPORTED),
+    (dict(block_size=24), psd.PS_ERR_UNSUPPORTED),
+    (dict(num_seqs=4097), psd.PS_ERR_UNSUPPORTED),
+    (dict(num_blocks=0), psd.PS_ERR_INVALID_ARG),
+    (dict(num_sms=-1), psd.PS_ERR_INVALID_ARG),
+])
+def test_plan_rejects_bad_shapes(kw, status):
+    with pytest.raises(psd.PsError) as ei:
+        _plan(**kw)
+    assert ei.value.status == status
+
+
+def test_calls_validate_before_touching_the_device():
+    plan, ws = _plan()
+    try:
+        # no workspace yet
+        with pytest.raises(psd.PsError) as ei:
+            psd.ps_decode_attention_planned(plan, 16, 16, 16, 16, 16, 16, 0.1, None)
+        assert ei.value.status == psd.PS_ERR_WORKSPACE
+        # null / misaligned pointers
+        with pytest.raises(psd.PsError) as ei:
+            psd.ps_decode_attention_planned(plan, 0, 16, 16, 16, 16, 16, 0.1, None)
+        assert ei.value.status == psd.PS_ERR_INVALID_ARG
+        with pytest.raises(psd.PsError) as ei:
+            psd.ps_decode_attention_planned(plan, 8, 16, 16, 16, 16, 16, 0.1, None)
+        assert ei.value.status == psd.PS_ERR_INVALID_ARG
+        with pytest.raises(psd.PsError) as ei:
+            psd.ps_decode_attention_planned(plan, 16, 16, 16, 16, 16, 16, float("nan"), None)
+        assert ei.value.status == psd.PS_ERR_INVALID_ARG
+        # workspace too small / misaligned
+        with pytest.raises(psd.PsError) as ei:
+            psd.ps_decode_plan_set_workspace(plan, 256, ws - 1)
+        assert ei.value.status == psd.PS_ERR_WORKSPACE
+        with pytest.raises(psd.PsError) as ei:
+            psd.ps_decode_plan_set_workspace(plan, 128, ws)
+        assert ei.value.status == psd.PS_ERR_INVALID_ARG
+    finally:
+        psd.ps_decode_plan_destroy(plan)
+
+
+def test_stream_binding_lookup():
+    plan, ws = _plan()
+    try:
+        fake_stream = 0x1234
+        # nothing bound to this stream
+        with pytest.raises(psd.PsError) as ei:
+            psd.ps_decode_attention(16, 16, 16, 16, 16, 16, 64, 32, 8, 128, 16, 0.1, fake_stream)
+        assert ei.value.status == psd.PS_ERR_NO_PLAN
+        psd.ps_decode_plan_bind(plan, fake_stream)
+        # bound, but the dims differ from the plan
+        with pytest.raises(psd.PsError) as ei:
+            psd.ps_decode_attention(16, 16, 16, 16, 16, 16, 64, 32, 8, 128, 32, 0.1, fake_stream)
+        assert ei.value.status == psd.PS_ERR_NO_PLAN
+        # bound and matching, but no workspace: fails before any CUDA call
+        with pytest.raises(psd.PsError) as ei:
+            psd.ps_decode_attention(16, 16, 16, 16, 16, 16, 64, 32, 8, 128, 16, 0.1, fake_stream)
+        assert ei.value.status == psd.PS_ERR_WORKSPACE
+        psd.ps_decode_plan_bind(None, fake_stream)
+        with pytest.raises(psd.PsError) as ei:
+            psd.ps_decode_attention(16, 16, 16, 16, 16, 16, 64, 32, 8, 128, 16, 0.1, fake_stream)
+        assert ei.value.status == psd.PS_ERR_NO_PLAN
+        psd.ps_decode_plan_bind(plan, fake_stream)
+    finally:
+        psd.ps_decode_plan_destroy(plan)
+    # destroying the plan dropped its binding
+    with pytest.raises(psd.PsError) as ei:
+        psd.ps_decode_attention(16, 16, 16, 16, 16, 16, 64, 32, 8, 128, 16, 0.1, 0x1234)
+    assert ei.value.status == psd.PS_ERR_NO_PLAN
+
+
+def test_worker_overrides_are_recorded():
+    plan, _ = _plan(max_workers=1, min_stages_per_worker=3)
+    try:
+        info = psd.ps_decode_plan_info(plan)
+        assert info["max_workers"] == 1 and info["min_stages_per_worker"] == 3
+    finally:
+        psd.ps_decode_plan_destroy(plan)

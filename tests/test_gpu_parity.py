@@ -1,0 +1,226 @@
+"""GPU parity: the CUDA path through the C ABI against the fp64 oracle.
+
+Tolerance (bf16 inputs drawn from N(0,1), bf16 output, scale 1/sqrt(128)):
+max |gpu - oracle| <= 8e-3 and mean |gpu - oracle| <= 1e-3 over every
+compared output element, and every output finite.
+
+Small cases compare every output; the four large workloads run at full
+size in the launch configuration the bench times and compare sampled
+sequences (shortest, longest and a few more) whose pages are copied back
+and fed to the oracle one by one.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_21719_gb300 import inputs
+
+pytestmark = pytest.mark.gpu
+
+MAX_ABS = 8e-3
+MEAN_ABS = 1e-3
+
+
+@pytest.fixture(scope="module")
+def psd():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2608_21719_gb300 import build
+    build.build()
+    from paper_2608_21719_gb300 import ps_decode
+    return ps_decode
+
+
+def _oracle(wl):
+    return oracle.decode_attention(inputs.bf16_bits(wl.q), inputs.bf16_bits(wl.k_cache),
+                                   inputs.bf16_bits(wl.v_cache), wl.block_table.cpu().numpy(),
+                                   wl.seq_lens.cpu().numpy(), wl.num_kv_heads, wl.scale)
+
+
+def _gpu(psd, wl, **kw):
+    attn = psd.DecodeAttention.for_workload(wl, **kw)
+    out = attn(wl.q, wl.k_cache, wl.v_cache, wl.block_table, wl.seq_lens, scale=wl.scale)
+    torch.cuda.synchronize()
+    status = attn.device_status()
+    info = attn.info()
+    attn.close()
+    return out, status, info
+
+
+def _compare(got, ref, what=""):
+    got = got.float().cpu().numpy().astype(np.float64)
+    assert np.all(np.isfinite(got)), "non-finite output %s" % what
+    err = np.abs(got - ref)
+    assert err.max() <= MAX_ABS, "%s max abs err %.3g" % (what, err.max())
+    assert err.mean() <= MEAN_ABS, "%s mean abs err %.3g" % (what, err.mean())
+    return err
+
+
+def _custom(Hq, Hkv, bs, lengths, seed, spare=5, device="cuda"):
+    lengths = np.asarray(lengths, dtype=np.int32)
+    mbps = max(1, (int(lengths.max(initial=0)) + bs - 1) // bs + 1)
+    nb = inputs.blocks_needed(lengths, bs) + spare
+    bt = inputs.build_block_table(lengths, bs, mbps, nb, np.random.default_rng(seed))
+    return inputs.make_tensors(Hq, Hkv, 128, bs, bt, lengths, nb, seed, device="cpu").to(device)
+
+
+def test_tiny_config_full_parity(psd):
+    wl = inputs.make_workload(1, device="cpu", spare_blocks=6).to("cuda")
+    out, status, _ = _gpu(psd, wl)
+    assert status == 0
+    _compare(out, _oracle(wl), "config 1")
+
+
+EDGE_LENGTHS = [1, 15, 16, 17, 31, 32, 33, 0, 47, 100, 1000]
+
+
+@pytest.mark.parametrize("Hq,Hkv", [(1, 1), (4, 2), (8, 2), (5, 1), (16, 2), (64, 8)])
+@pytest.mark.parametrize("bs", [16, 32, 64])
+def test_edge_lengths_groups_and_block_sizes(psd, Hq, Hkv, bs):
+    wl = _custom(Hq, Hkv, bs, EDGE_LENGTHS, seed=Hq * 100 + bs)
+    out, status, _ = _gpu(psd, wl)
+    assert status == 0
+    ref = _oracle(wl)
+    _compare(out, ref, "edge Hq=%d Hkv=%d bs=%d" % (Hq, Hkv, bs))
+    assert torch.all(out[7] == 0)  # empty sequence
+
+
+@pytest.mark.parametrize("max_workers,min_stages", [(1, 0), (2, 1), (7, 1), (0, 1), (0, 3), (0, 0), (33, 2)])
+def test_forced_splits(psd, max_workers, min_stages):
+    wl = _custom(32, 8, 16, [1, 200, 513, 16, 2049, 37, 777, 64], seed=5)
+    out, status, info = _gpu(psd, wl, max_workers=max_workers, min_stages_per_worker=min_stages)
+    assert status == 0
+    _compare(out, _oracle(wl), "split %s/%s" % (max_workers, min_stages))
+
+
+def test_single_token_returns_value_row_exactly(psd):
+    wl = _custom(8, 2, 16, [1, 1, 1, 1], seed=9)
+    out, status, _ = _gpu(psd, wl)
+    for s in range(4):
+        b = int(wl.block_table[s, 0])
+        for h in range(8):
+            assert torch.equal(out[s, h], wl.v_cache[b, h // 4, 0])
+
+
+def test_constant_values_return_that_value(psd):
+    wl = _custom(32, 8, 16, [5, 300, 4000], seed=10)
+    wl.v_cache.fill_(0.8125)
+    out, status, _ = _gpu(psd, wl)
+    assert torch.all(out.float() == 0.8125)
+
+
+def test_deterministic_and_relabelling_invariant(psd):
+    lengths = np.array([900, 31, 2000, 1, 64, 513], dtype=np.int32)
+    bs, Hq, Hkv = 16, 32, 8
+    wl = _custom(Hq, Hkv, bs, lengths, seed=12, spare=11)
+    out1, _, _ = _gpu(psd, wl)
+    out2, _, _ = _gpu(psd, wl)
+    assert torch.equal(out1, out2)
+    # Same logical tokens, different physical blocks.
+    nb = wl.num_blocks
+    bt2 = inputs.build_block_table(lengths, bs, wl.max_blocks_per_seq, nb, np.random.default_rng(77))
+    bt1 = wl.block_table.cpu().numpy()
+    k2 = torch.full_like(wl.k_cache, float("nan"))
+    v2 = torch.full_like(wl.v_cache, float("nan"))
+    for s, L in enumerate(lengths):
+        n = (int(L) + bs - 1) // bs
+        src = torch.from_numpy(bt1[s, :n]).long().cuda()
+        dst = torch.from_numpy(bt2[s, :n]).long().cuda()
+        k2[dst] = wl.k_cache[src]
+        v2[dst] = wl.v_cache[src]
+    wl2 = inputs.Workload(cfg=None, q=wl.q, k_cache=k2, v_cache=v2,
+                          block_table=torch.from_numpy(bt2).cuda(), seq_lens=wl.seq_lens, scale=wl.scale)
+    out3, _, _ = _gpu(psd, wl2)
+    assert torch.equal(out1, out3)
+
+
+def test_thirteen_argument_call_uses_the_bound_plan(psd):
+    wl = _custom(8, 2, 32, [40, 500, 3], seed=13)
+    plan, ws = psd.ps_decode_plan_create(wl.num_seqs, wl.num_q_heads, wl.num_kv_heads, 128, wl.block_size,
+                                         wl.max_blocks_per_seq, wl.num_blocks)
+    work = torch.empty(ws, dtype=torch.uint8, device="cuda")
+    psd.ps_decode_plan_set_workspace(plan, work, ws)
+    stream = torch.cuda.Stream()
+    psd.ps_decode_plan_bind(plan, stream)
+    out = torch.empty_like(wl.q)
+    with torch.cuda.stream(stream):
+        psd.ps_decode_attention(wl.q, wl.k_cache, wl.v_cache, wl.block_table, wl.seq_lens, out, wl.num_seqs,
+                                wl.num_q_heads, wl.num_kv_heads, 128, wl.block_size, wl.scale, stream)
+    stream.synchronize()
+    with pytest.raises(psd.PsError) as ei:  # nothing bound to the default stream
+        psd.ps_decode_attention(wl.q, wl.k_cache, wl.v_cache, wl.block_table, wl.seq_lens, out, wl.num_seqs,
+                                wl.num_q_heads, wl.num_kv_heads, 128, wl.block_size, wl.scale, None)
+    assert ei.value.status == psd.PS_ERR_NO_PLAN
+    psd.ps_decode_plan_destroy(plan)
+    _compare(out, _oracle(wl), "13-arg")
+
+
+def test_timing_events_are_recorded(psd):
+    wl = _custom(32, 8, 16, [3000, 4000], seed=14)
+    attn = psd.DecodeAttention.for_workload(wl)
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+    psd.ps_decode_plan_set_timing_events(attn.plan, *evs)
+    n0 = psd.ps_decode_launch_count()
+    attn(wl.q, wl.k_cache, wl.v_cache, wl.block_table, wl.seq_lens)
+    torch.cuda.synchronize()
+    assert psd.ps_decode_launch_count() - n0 == 2
+    assert evs[0].elapsed_time(evs[1]) > 0 and evs[1].elapsed_time(evs[2]) > 0
+    attn.close()
+
+
+def test_bad_block_id_and_overlong_length_raise_device_flags(psd):
+    wl = _custom(8, 2, 16, [40, 70], seed=15)
+    bt = wl.block_table.clone()
+    bt[1, 2] = wl.num_blocks + 5  # outside the pool: the kernel reads zeros and flags it
+    wl_bad = inputs.Workload(cfg=None, q=wl.q, k_cache=wl.k_cache, v_cache=wl.v_cache, block_table=bt,
+                             seq_lens=wl.seq_lens, scale=wl.scale)
+    out, status, _ = _gpu(psd, wl_bad)
+    assert status & psd.PS_DEVICE_BAD_BLOCK
+    assert torch.all(torch.isfinite(out.float()))
+    sl = wl.seq_lens.clone()
+    sl[0] = wl.max_blocks_per_seq * 16 + 100  # longer than its block-table row: clamped
+    bt2 = wl.block_table.clone()
+    bt2[0] = torch.arange(wl.max_blocks_per_seq, device="cuda", dtype=torch.int32) % wl.num_blocks
+    wl_long = inputs.Workload(cfg=None, q=wl.q, k_cache=torch.nan_to_num(wl.k_cache),
+                              v_cache=torch.nan_to_num(wl.v_cache), block_table=bt2, seq_lens=sl, scale=wl.scale)
+    out, status, _ = _gpu(psd, wl_long)
+    assert status & psd.PS_DEVICE_LEN_CLAMPED
+    assert torch.all(torch.isfinite(out.float()))
+
+
+def _sampled_rows(wl, idx):
+    """Copy the pages of sequences ``idx`` back to the host as a compact workload."""
+    bs = wl.block_size
+    lens = wl.seq_lens[idx].cpu().numpy()
+    bt = wl.block_table[idx].cpu().numpy()
+    pages = [bt[i, :(int(L) + bs - 1) // bs] for i, L in enumerate(lens)]
+    flat = torch.from_numpy(np.concatenate(pages).astype(np.int64)).cuda()
+    k = wl.k_cache.index_select(0, flat).cpu()
+    v = wl.v_cache.index_select(0, flat).cpu()
+    nbt = np.full((len(idx), max(1, max(len(p) for p in pages))), -1, dtype=np.int32)
+    pos = 0
+    for i, p in enumerate(pages):
+        nbt[i, :len(p)] = np.arange(pos, pos + len(p))
+        pos += len(p)
+    return inputs.Workload(cfg=None, q=wl.q[idx].cpu(), k_cache=k, v_cache=v, block_table=torch.from_numpy(nbt),
+                           seq_lens=torch.from_numpy(lens.astype(np.int32)), scale=wl.scale)
+
+
+@pytest.mark.parametrize("key", [2, 3, 4, 5])
+def test_full_size_configs_sampled(psd, key):
+    wl = inputs.make_workload(key, device="cuda", poison=True)
+    out, status, info = _gpu(psd, wl)
+    assert status == 0
+    assert torch.all(torch.isfinite(out.float()))
+    lens = wl.seq_lens.cpu().numpy()
+    order = np.argsort(lens)
+    rng = np.random.default_rng(key)
+    idx = sorted(set([int(order[0]), int(order[-1]), int(order[len(order) // 2])] +
+                     [int(i) for i in rng.choice(len(lens), size=min(3, len(lens)), replace=False)]))
+    sub = _sampled_rows(wl, idx)
+    _compare(out[idx], _oracle(sub), "config %d sampled %s" % (key, idx))
+    del wl
+    torch.cuda.empty_cache()
