@@ -50,11 +50,20 @@ def _gpu(psd, wl, **kw):
     return out, status, info
 
 
-def _compare(got, ref, what=""):
+# Short contexts average few value rows, so |o| reaches 2-4 and the bf16
+# output rounding alone (relative error <= 2^-8) exceeds 8e-3 there.  Custom
+# edge cases therefore allow that rounding term on top of the absolute bound;
+# the five named workloads are held to the plain bounds.
+BF16_REL = 2.0 ** -8
+
+
+def _compare(got, ref, what="", rel=BF16_REL):
     got = got.float().cpu().numpy().astype(np.float64)
     assert np.all(np.isfinite(got)), "non-finite output %s" % what
     err = np.abs(got - ref)
-    assert err.max() <= MAX_ABS, "%s max abs err %.3g" % (what, err.max())
+    excess = err - (MAX_ABS + rel * np.abs(ref))
+    assert excess.max() <= 0, "%s max abs err %.3g (at |ref| %.3g)" % (
+        what, err.max(), np.abs(ref).flat[int(np.argmax(excess))])
     assert err.mean() <= MEAN_ABS, "%s mean abs err %.3g" % (what, err.mean())
     return err
 
@@ -71,7 +80,7 @@ def test_tiny_config_full_parity(psd):
     wl = inputs.make_workload(1, device="cpu", spare_blocks=6).to("cuda")
     out, status, _ = _gpu(psd, wl)
     assert status == 0
-    _compare(out, _oracle(wl), "config 1")
+    _compare(out, _oracle(wl), "config 1", rel=0.0)
 
 
 EDGE_LENGTHS = [1, 15, 16, 17, 31, 32, 33, 0, 47, 100, 1000]
@@ -221,6 +230,6 @@ def test_full_size_configs_sampled(psd, key):
     idx = sorted(set([int(order[0]), int(order[-1]), int(order[len(order) // 2])] +
                      [int(i) for i in rng.choice(len(lens), size=min(3, len(lens)), replace=False)]))
     sub = _sampled_rows(wl, idx)
-    _compare(out[idx], _oracle(sub), "config %d sampled %s" % (key, idx))
+    _compare(out[idx], _oracle(sub), "config %d sampled %s" % (key, idx), rel=0.0)
     del wl
     torch.cuda.empty_cache()
