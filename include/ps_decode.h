@@ -27,9 +27,8 @@
  *
  * ----------------------------------------------------------- conventions --
  *  - Every tensor pointer is a DEVICE pointer owned by the caller; the library
- *    never allocates or frees device memory.  q, k_cache and v_cache must be
- *    16-byte aligned; block_table and seq_lens 4-byte aligned; out 2-byte
- *    aligned.
+ *    never allocates or frees device memory.  q, k_cache, v_cache and out
+ *    must be 16-byte aligned; block_table and seq_lens 4-byte aligned.
  *  - Calls are asynchronous and ordered on the given CUDA stream
  *    (cudaStream_t passed as void*; NULL is the legacy default stream).
  *  - Supported shapes: head_dim == 128; 1 <= num_q_heads / num_kv_heads <= 8;
@@ -40,8 +39,14 @@
  *    outside [0, num_blocks) reads zeros; both set a flag readable with
  *    ps_decode_plan_read_device_status().  Nothing faults.
  *  - Split-KV workspace: the caller allocates ps_decode_plan_create()'s
- *    workspace_bytes of device memory and hands it to the plan.  One
- *    workspace must not be used by two calls that can run concurrently.
+ *    workspace_bytes of device memory and hands it to the plan.  It holds
+ *    the partial (max, sum, weighted-value) states of cut pieces plus a few
+ *    counters that every call leaves at zero.  One workspace must not be
+ *    used by two calls that can run concurrently; after a call that raised
+ *    PS_DEVICE_TIMEOUT, hand the workspace to the plan again
+ *    (ps_decode_plan_set_workspace) so that its counters are re-zeroed.
+ *  - Results are deterministic: the split of the work depends only on the
+ *    sequence lengths and the plan, never on scheduling.
  *  - A plan is not thread-safe: use it from one host thread at a time.
  */
 #ifndef PS_DECODE_H
@@ -78,17 +83,18 @@ typedef struct ps_decode_plan_info {
     int grid_ctas;             /* CTAs of the split-KV partial kernel */
     int workers_per_cta;       /* independent streaming warps per CTA */
     int stages_per_worker;     /* 16-token K/V tiles in flight per warp */
-    int max_workers;           /* cap on the balanced partition's worker count */
-    int min_stages_per_worker; /* floor on a worker's share, in 16-token tiles */
+    int max_workers;           /* cap on the static partition's worker count */
+    int min_stages_per_worker; /* floor on a static worker's share, in 16-token tiles */
+    int dynamic_permille;      /* share of the work handed out as dynamic chunks */
     size_t workspace_bytes;
     size_t smem_bytes;         /* dynamic shared memory of the partial kernel */
 } ps_decode_plan_info_t;
 
 /*
- * Plan a decode-attention shape.  The plan fixes the grid of the split-KV
- * partial kernel (one CTA per SM) and sizes the workspace that carries the
- * per-worker partial (max, sum, weighted-value) states to the log-sum-exp
- * combine.  No device memory is allocated.
+ * Plan a decode-attention shape.  The plan fixes the grid of the kernel (one
+ * CTA per SM, eight streaming warps each) and sizes the workspace that
+ * carries the partial (max, sum, weighted-value) states of split-KV pieces
+ * to the log-sum-exp merge.  No device memory is allocated.
  *
  *   max_blocks_per_seq  row stride of block_table (entries)
  *   num_blocks          physical blocks in k_cache / v_cache (TMA bounds)
@@ -105,23 +111,30 @@ ps_status_t ps_decode_plan_create(int num_seqs, int num_q_heads, int num_kv_head
                                   ps_decode_plan_t **plan, size_t *workspace_bytes);
 
 /*
- * As ps_decode_plan_create(), with explicit knobs (0 = default for each):
+ * As ps_decode_plan_create(), with explicit knobs (0 = default for the first
+ * three, -1 = default for dynamic_permille):
  *   num_sms                SM count to size the grid for (0: query the device;
  *                          a positive value needs no GPU, e.g. for host tests)
- *   max_workers            upper bound on the number of balanced workers the
- *                          kernel splits the batch's KV stream into
- *                          (1 = no split at all)
- *   min_stages_per_worker  smallest share of a worker, in 16-token tiles
+ *   max_workers            upper bound on the number of equal static ranges
+ *                          the batch's KV stream is split into
+ *   min_stages_per_worker  smallest static range, in 16-token tiles
  *                          (1 = split as finely as the workers allow)
+ *   dynamic_permille       share (0..1000) of the KV stream cut into small
+ *                          fixed chunks that idle warps claim at run time;
+ *                          0 = fully static split, -1 = default (0)
+ * max_workers = 1 with dynamic_permille = 0 runs the whole batch in one
+ * warp without any split.
  */
 ps_status_t ps_decode_plan_create_ex(int num_seqs, int num_q_heads, int num_kv_heads, int head_dim,
                                      int block_size, int max_blocks_per_seq, long long num_blocks,
                                      int num_sms, int max_workers, int min_stages_per_worker,
-                                     ps_decode_plan_t **plan, size_t *workspace_bytes);
+                                     int dynamic_permille, ps_decode_plan_t **plan,
+                                     size_t *workspace_bytes);
 
 /* Give the plan its caller-owned device workspace (>= workspace_bytes, 256-byte
- * aligned).  The first call after this zeroes the workspace's status word on
- * that call's stream.  Errors: PS_ERR_INVALID_ARG, PS_ERR_WORKSPACE. */
+ * aligned).  The first call after this zeroes the workspace's counters and
+ * status word on that call's stream.  Errors: PS_ERR_INVALID_ARG,
+ * PS_ERR_WORKSPACE. */
 ps_status_t ps_decode_plan_set_workspace(ps_decode_plan_t *plan, void *workspace, size_t bytes);
 
 /* Bind the plan to a stream so that ps_decode_attention() on that stream
@@ -139,9 +152,10 @@ ps_status_t ps_decode_plan_info(const ps_decode_plan_t *plan, ps_decode_plan_inf
 
 /*
  * Decode attention with the plan bound to `stream` (ps_decode_plan_bind).
- * Launches the split-KV partial kernel and the log-sum-exp combine kernel on
- * `stream`.  scale is applied to q . k before the softmax (1/sqrt(head_dim)
- * for standard attention; any finite value is accepted).
+ * Launches one kernel on `stream`: the split-KV streaming pass with the
+ * log-sum-exp merge of cut pieces fused into it.  scale is applied to q . k
+ * before the softmax (1/sqrt(head_dim) for standard attention; any finite
+ * value is accepted).
  *
  * Errors: PS_ERR_NO_PLAN when no plan is bound to `stream` or its
  * (num_seqs, num_q_heads, num_kv_heads, head_dim, block_size) differ from the
@@ -162,12 +176,10 @@ ps_status_t ps_decode_attention_planned(const ps_decode_plan_t *plan, const void
 
 /*
  * Measurement hook: when events are set (cudaEvent_t as void*, NULL to
- * clear), every call records ev_start before the partial kernel, ev_mid
- * between the partial and the combine kernel, and ev_end after the combine,
- * on the call's stream.
+ * clear), every call records ev_start right before its kernel and ev_end
+ * right after it, on the call's stream.
  */
-ps_status_t ps_decode_plan_set_timing_events(ps_decode_plan_t *plan, void *ev_start, void *ev_mid,
-                                             void *ev_end);
+ps_status_t ps_decode_plan_set_timing_events(ps_decode_plan_t *plan, void *ev_start, void *ev_end);
 
 /* Copy the device status word (PS_DEVICE_* flags raised by calls since the
  * last read) to *flags, synchronising `stream`, then clear it.  Errors:

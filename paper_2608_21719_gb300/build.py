@@ -34,6 +34,7 @@ def nvcc() -> str:
 
 def _flags(verbose: bool) -> list:
     f = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I", INCLUDE, "-I", CSRC]
+    f += os.environ.get("PS_NVCC_FLAGS", "").split()
     if verbose:
         f += ["-Xptxas", "-v"]
     return f

@@ -1,5 +1,5 @@
 // ps_decode_host.cpp -- the C ABI of include/ps_decode.h: argument checks,
-// plans, stream bindings, TMA descriptor encoding and the two launches.
+// plans, stream bindings, TMA descriptor encoding and the launch.
 #include <cuda.h>
 #include <cuda_runtime.h>
 
@@ -20,7 +20,7 @@ struct ps_decode_plan {
     uint32_t magic;
     int num_seqs, num_q_heads, num_kv_heads, head_dim, block_size, max_blocks_per_seq;
     long long num_blocks;
-    int num_sms, grid_ctas, max_workers, min_stages;
+    int num_sms, grid_ctas, max_workers, min_stages, dynamic_permille;
     size_t smem_bytes;
     WorkspaceLayout ws;
     void *workspace = nullptr;
@@ -30,7 +30,7 @@ struct ps_decode_plan {
     const void *tm_k_ptr = nullptr, *tm_v_ptr = nullptr;
     alignas(64) CUtensorMap tmK;
     alignas(64) CUtensorMap tmV;
-    cudaEvent_t ev_start = nullptr, ev_mid = nullptr, ev_end = nullptr;
+    cudaEvent_t ev_start = nullptr, ev_end = nullptr;
 };
 
 namespace {
@@ -101,7 +101,7 @@ ps_status_t run_planned(ps_decode_plan *p, const void *q, const void *k, const v
                         const int *sl, void *out, float scale, void *stream) {
     if (!q || !k || !v || !bt || !sl || !out) return PS_ERR_INVALID_ARG;
     if (!aligned(q, 16) || !aligned(k, 16) || !aligned(v, 16) || !aligned(bt, 4) || !aligned(sl, 4) ||
-        !aligned(out, 2))
+        !aligned(out, 16))
         return PS_ERR_INVALID_ARG;
     if (!std::isfinite(scale)) return PS_ERR_INVALID_ARG;
     if (!p->workspace || p->workspace_size < p->ws.total) return PS_ERR_WORKSPACE;
@@ -119,47 +119,36 @@ ps_status_t run_planned(ps_decode_plan *p, const void *q, const void *k, const v
     }
     uint8_t *ws = static_cast<uint8_t *>(p->workspace);
     if (p->status_needs_clear) {
-        if (cudaMemsetAsync(ws, 0, kWsHeaderBytes, st) != cudaSuccess) return PS_ERR_CUDA;
+        // Status word, chunk dispenser and per-segment counters start at zero;
+        // the kernel returns them to zero at the end of every call.
+        if (cudaMemsetAsync(ws, 0, p->ws.acc_off, st) != cudaSuccess) return PS_ERR_CUDA;
         p->status_needs_clear = false;
     }
 
-    PartialParams pp;
-    pp.q = static_cast<const uint16_t *>(q);
-    pp.block_table = bt;
-    pp.seq_lens = sl;
-    pp.out = static_cast<uint16_t *>(out);
-    pp.ws_header = reinterpret_cast<int *>(ws);
-    pp.ws_prefix = reinterpret_cast<int *>(ws + p->ws.prefix_off);
-    pp.ws_acc = reinterpret_cast<float *>(ws + p->ws.acc_off);
-    pp.ws_ml = reinterpret_cast<float *>(ws + p->ws.ml_off);
-    pp.num_seqs = p->num_seqs;
-    pp.num_q_heads = p->num_q_heads;
-    pp.num_kv_heads = p->num_kv_heads;
-    pp.group = p->num_q_heads / p->num_kv_heads;
-    pp.block_size = p->block_size;
-    pp.max_blocks_per_seq = p->max_blocks_per_seq;
-    pp.num_blocks = p->num_blocks;
-    pp.len_cap = p->max_blocks_per_seq * p->block_size;
-    pp.max_workers = p->max_workers;
-    pp.min_stages = p->min_stages;
-    pp.scale_log2 = (float)((double)scale * 1.4426950408889634);
-
-    CombineParams cp;
-    cp.out = pp.out;
-    cp.ws_header = pp.ws_header;
-    cp.ws_prefix = pp.ws_prefix;
-    cp.ws_acc = pp.ws_acc;
-    cp.ws_ml = pp.ws_ml;
-    cp.num_seqs = pp.num_seqs;
-    cp.num_q_heads = pp.num_q_heads;
-    cp.num_kv_heads = pp.num_kv_heads;
-    cp.group = pp.group;
+    DecodeParams dp;
+    dp.q = static_cast<const uint16_t *>(q);
+    dp.block_table = bt;
+    dp.seq_lens = sl;
+    dp.out = static_cast<uint16_t *>(out);
+    dp.ws_header = reinterpret_cast<int *>(ws);
+    dp.seg_done = reinterpret_cast<int *>(ws + p->ws.seg_done_off);
+    dp.ws_acc = reinterpret_cast<float *>(ws + p->ws.acc_off);
+    dp.ws_ml = reinterpret_cast<float *>(ws + p->ws.ml_off);
+    dp.num_seqs = p->num_seqs;
+    dp.num_q_heads = p->num_q_heads;
+    dp.num_kv_heads = p->num_kv_heads;
+    dp.group = p->num_q_heads / p->num_kv_heads;
+    dp.block_size = p->block_size;
+    dp.max_blocks_per_seq = p->max_blocks_per_seq;
+    dp.num_blocks = p->num_blocks;
+    dp.len_cap = p->max_blocks_per_seq * p->block_size;
+    dp.max_workers = p->max_workers;
+    dp.min_stages = p->min_stages;
+    dp.dynamic_permille = p->dynamic_permille;
+    dp.scale_log2 = (float)((double)scale * 1.4426950408889634);
 
     if (p->ev_start && cudaEventRecord(p->ev_start, st) != cudaSuccess) return PS_ERR_CUDA;
-    if (launch_partial(pp, p->tmK, p->tmV, p->grid_ctas, p->smem_bytes, st) != cudaSuccess) return PS_ERR_CUDA;
-    g_launches.fetch_add(1, std::memory_order_relaxed);
-    if (p->ev_mid && cudaEventRecord(p->ev_mid, st) != cudaSuccess) return PS_ERR_CUDA;
-    if (launch_combine(cp, st) != cudaSuccess) return PS_ERR_CUDA;
+    if (launch_decode(dp, p->tmK, p->tmV, p->grid_ctas, p->smem_bytes, st) != cudaSuccess) return PS_ERR_CUDA;
     g_launches.fetch_add(1, std::memory_order_relaxed);
     if (p->ev_end && cudaEventRecord(p->ev_end, st) != cudaSuccess) return PS_ERR_CUDA;
     return PS_OK;
@@ -171,11 +160,14 @@ extern "C" {
 
 ps_status_t ps_decode_plan_create_ex(int num_seqs, int num_q_heads, int num_kv_heads, int head_dim, int block_size,
                                      int max_blocks_per_seq, long long num_blocks, int num_sms, int max_workers,
-                                     int min_stages_per_worker, ps_decode_plan_t **plan, size_t *workspace_bytes) {
+                                     int min_stages_per_worker, int dynamic_permille, ps_decode_plan_t **plan,
+                                     size_t *workspace_bytes) {
     if (!plan || !workspace_bytes) return PS_ERR_INVALID_ARG;
     *plan = nullptr;
     *workspace_bytes = 0;
-    if (num_sms < 0 || max_workers < 0 || min_stages_per_worker < 0) return PS_ERR_INVALID_ARG;
+    if (num_sms < 0 || max_workers < 0 || min_stages_per_worker < 0 || dynamic_permille < -1 ||
+        dynamic_permille > 1000)
+        return PS_ERR_INVALID_ARG;
     ps_status_t e = check_shape(num_seqs, num_q_heads, num_kv_heads, head_dim, block_size, max_blocks_per_seq,
                                 num_blocks);
     if (e != PS_OK) return e;
@@ -200,8 +192,9 @@ ps_status_t ps_decode_plan_create_ex(int num_seqs, int num_q_heads, int num_kv_h
     const int total_workers = p->grid_ctas * kWorkersPerCta;
     p->max_workers = (max_workers > 0 && max_workers < total_workers) ? max_workers : total_workers;
     p->min_stages = min_stages_per_worker > 0 ? min_stages_per_worker : kDefaultMinStages;
+    p->dynamic_permille = dynamic_permille >= 0 ? dynamic_permille : kDefaultDynamicPermille;
     p->smem_bytes = partial_smem_bytes(num_seqs);
-    p->ws = workspace_layout(num_seqs, total_workers);
+    p->ws = workspace_layout(num_seqs, num_kv_heads, total_workers);
     *plan = p;
     *workspace_bytes = p->ws.total;
     return PS_OK;
@@ -211,7 +204,7 @@ ps_status_t ps_decode_plan_create(int num_seqs, int num_q_heads, int num_kv_head
                                   int max_blocks_per_seq, long long num_blocks, ps_decode_plan_t **plan,
                                   size_t *workspace_bytes) {
     return ps_decode_plan_create_ex(num_seqs, num_q_heads, num_kv_heads, head_dim, block_size, max_blocks_per_seq,
-                                    num_blocks, 0, 0, 0, plan, workspace_bytes);
+                                    num_blocks, 0, 0, 0, -1, plan, workspace_bytes);
 }
 
 ps_status_t ps_decode_plan_set_workspace(ps_decode_plan_t *plan, void *workspace, size_t bytes) {
@@ -262,6 +255,7 @@ ps_status_t ps_decode_plan_info(const ps_decode_plan_t *plan, ps_decode_plan_inf
     info->stages_per_worker = kStages;
     info->max_workers = plan->max_workers;
     info->min_stages_per_worker = plan->min_stages;
+    info->dynamic_permille = plan->dynamic_permille;
     info->workspace_bytes = plan->ws.total;
     info->smem_bytes = plan->smem_bytes;
     return PS_OK;
@@ -291,10 +285,9 @@ ps_status_t ps_decode_attention(const void *q, const void *k_cache, const void *
     return run_planned(p, q, k_cache, v_cache, block_table, seq_lens, out, scale, stream);
 }
 
-ps_status_t ps_decode_plan_set_timing_events(ps_decode_plan_t *plan, void *ev_start, void *ev_mid, void *ev_end) {
+ps_status_t ps_decode_plan_set_timing_events(ps_decode_plan_t *plan, void *ev_start, void *ev_end) {
     if (!live(plan)) return PS_ERR_INVALID_ARG;
     plan->ev_start = reinterpret_cast<cudaEvent_t>(ev_start);
-    plan->ev_mid = reinterpret_cast<cudaEvent_t>(ev_mid);
     plan->ev_end = reinterpret_cast<cudaEvent_t>(ev_end);
     return PS_OK;
 }

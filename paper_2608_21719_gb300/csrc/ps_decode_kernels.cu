@@ -1,31 +1,37 @@
-// ps_decode_kernels.cu -- sm_103a kernels for batched paged GQA decode attention.
+// ps_decode_kernels.cu -- sm_103a kernel for batched paged GQA decode attention.
 //
-// Two launches per call:
+// One persistent launch per call: one CTA per SM, kWorkersPerCta independent
+// worker warps per CTA.
 //
-//  1. ps_decode_partial_kernel (persistent, one CTA per SM, 4 independent
-//     worker warps per CTA).  The KV work of the whole batch is laid out as
-//     one "tape" of 16-token tiles, ordered by sequence and then KV head:
-//     segment (s, j) holds ceil(L_s / 16) tiles.  Every CTA rebuilds the
-//     per-sequence prefix sums of that tape in shared memory, and worker w of
-//     W gets the contiguous range [floor(w N / W), floor((w+1) N / W)) of the
-//     N tiles.  The split is therefore balanced to one tile whatever the mix
-//     of short answer-phase and long thinking-phase contexts (PowerSlider
-//     Sec. 2.2, Sec. 3 Obs. 3), with no atomics and no host knowledge of the
-//     lengths.  A worker streams its tiles through a ring of shared-memory
-//     stages filled by TMA (cp.async.bulk.tensor, 128-byte swizzle) and
-//     completed on mbarriers, reading each (block, kv-head) page exactly
-//     once for all g query heads of the group.  Per tile it computes the
-//     scores S^T = K Q^T and the update O^T += V^T P^T on the tensor cores
-//     (mma.sync m16n8k16, bf16 in, fp32 accumulate: tokens fill M = 16, the
-//     g <= 8 heads of the group fill N = 8), with an online softmax whose
-//     running max and sum stay in fp32.  A piece of a segment that a worker
-//     covers completely is normalised and written as bf16 output; a piece cut
-//     by a worker boundary leaves (m, l, acc) in the workspace.
+// Work layout.  The KV work of the whole batch is one "tape" of 16-token
+// tiles ordered by sequence, then KV head: segment (s, j) holds
+// ceil(L_s / 16) tiles.  Every CTA rebuilds the per-sequence prefix sums of
+// the tape in shared memory.  The first part of the tape is split into equal
+// contiguous static ranges, one per worker; the last part
+// (dynamic_permille / 1000 of it) is cut into fixed chunks that idle workers
+// claim from an atomic dispenser, so random per-SM and per-warp speed
+// differences are absorbed at the end instead of stretching the tail.  All
+// range boundaries are a fixed function of the lengths and the grid, so the
+// result does not depend on which warp ran which range.  The mix of short
+// answer-phase and long thinking-phase contexts (PowerSlider Sec. 2.2, Sec. 3
+// Obs. 3) therefore needs no host knowledge of the lengths.
 //
-//  2. ps_decode_combine_kernel merges the pieces of every cut segment with
-//     the log-sum-exp rule o = sum_c 2^(m_c - M) acc_c / sum_c 2^(m_c - M) l_c
-//     (scores are kept in base 2 with log2(e) folded into the scale), and
-//     zero-fills the rows of empty sequences.
+// Streaming.  A worker walks its ranges tile by tile.  Each tile's K and V
+// page halves arrive by TMA (cp.async.bulk.tensor, 128-byte swizzle) in a
+// per-warp ring of shared-memory stages completed on mbarriers; each
+// (block, kv-head) page is read once for all g query heads of its group.
+// Per tile the warp computes S^T = K Q^T and O^T += V^T P^T on the tensor
+// cores (mma.sync m16n8k16, bf16 in, fp32 accumulate: tokens fill M = 16,
+// the g <= 8 query heads fill N = 8) with an online softmax whose running
+// max and sum stay in fp32 (scores in base 2, log2(e) folded into scale).
+//
+// Split-KV combine.  A piece of a segment that one range covers completely
+// is normalised and written as bf16.  A piece cut by a range boundary leaves
+// (m, l, acc) in the workspace and adds its tile count to the segment's
+// counter; the warp that completes the count merges all pieces of the
+// segment in tape order by the log-sum-exp rule
+//   o = sum_c 2^(m_c - M) acc_c / sum_c 2^(m_c - M) l_c,  M = max_c m_c,
+// and resets the counter for the next call.
 //
 // No wait spins forever: every mbarrier wait gives up after ~2 s of
 // globaltimer, raises PS_DEVICE_TIMEOUT in the workspace status word, drains
@@ -108,6 +114,10 @@ __device__ __forceinline__ void bulk_load(uint32_t dst, const void *src, uint32_
         : "memory");
 }
 
+__device__ __forceinline__ void prefetch_l2(const void *p) {
+    asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
+}
+
 __device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3) {
     asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
                  : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
@@ -171,7 +181,7 @@ struct Cursor {
 
 __device__ __forceinline__ int tiles_of(int len) { return (len + kTileTokens - 1) / kTileTokens; }
 
-__device__ __forceinline__ Cursor locate(const int *sP, const int *sL, int S, int Hkv, int x) {
+__device__ __forceinline__ Cursor locate(const int *sP, const int *sL, int S, int x) {
     int lo = 0, hi = S - 1;
     while (lo < hi) {
         const int mid = (lo + hi + 1) >> 1;
@@ -183,7 +193,6 @@ __device__ __forceinline__ Cursor locate(const int *sP, const int *sL, int S, in
     const int off = x - sP[lo];
     c.h = off / c.ns;
     c.st = off - c.h * c.ns;
-    (void)Hkv;
     return c;
 }
 
@@ -198,23 +207,132 @@ __device__ __forceinline__ void advance(Cursor &c, const int *sL, int S, int Hkv
     c.ns = c.s < S ? tiles_of(sL[c.s]) : 0;
 }
 
-// ------------------------------------------------------ partial kernel ----
+// Split of the tape into static worker ranges followed by dynamic chunks.
+// Range ids: static ranges 0 .. Ws-1, dynamic chunks Ws .. Ws+K-1, in tape order.
+struct Partition {
+    int N, Ns, Ws, Cd, K;
+
+    __device__ int range_of(int x) const {
+        if (x < Ns) return (int)((((long long)x + 1) * Ws - 1) / Ns);
+        return Ws + (x - Ns) / Cd;
+    }
+    __device__ int range_begin(int r) const {
+        if (r < Ws) return (int)((long long)r * Ns / Ws);
+        return Ns + (r - Ws) * Cd;
+    }
+    __device__ int range_end(int r) const {
+        if (r < Ws) return (int)((long long)(r + 1) * Ns / Ws);
+        return min(N, Ns + (r - Ws + 1) * Cd);
+    }
+};
+
+// Merge every cut piece of segment (s, h) in tape order into bf16 output rows.
+// Pieces are read through L2 (other SMs wrote them).  Lanes take one piece
+// each for the (m, l) pass; for the weighted sum every lane owns dims
+// [4*lane, 4*lane+4) of every head, so all loads of a piece are in flight
+// together.
+__device__ void merge_segment(const DecodeParams &p, const Partition &part, int a, int b, int s, int h, int lane) {
+    const int g = p.group;
+    const int r0 = part.range_of(a), r1 = part.range_of(b - 1);
+    auto slot_of = [&](int r) -> size_t { return 2 * (size_t)r + (part.range_begin(r) < a ? 1 : 0); };
+    // Pass 1: per-head maximum over all pieces of their running maxima.
+    float M[kMaxGroup];
+#pragma unroll
+    for (int n = 0; n < kMaxGroup; ++n) M[n] = -INFINITY;
+    for (int r = r0 + lane; r <= r1; r += 32) {
+        const float4 *ml = reinterpret_cast<const float4 *>(p.ws_ml + slot_of(r) * kSlotMl);
+#pragma unroll
+        for (int q4 = 0; q4 < kMaxGroup / 2; ++q4) {
+            const float4 v = __ldcg(ml + q4);
+            M[2 * q4] = fmaxf(M[2 * q4], v.x);
+            M[2 * q4 + 1] = fmaxf(M[2 * q4 + 1], v.z);
+        }
+    }
+#pragma unroll
+    for (int n = 0; n < kMaxGroup; ++n)
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) M[n] = fmaxf(M[n], __shfl_xor_sync(kFull, M[n], o));
+    // Pass 2: weights per piece and head, weighted sums of the pieces.
+    float4 acc[kMaxGroup];
+    float lsum[kMaxGroup];
+#pragma unroll
+    for (int n = 0; n < kMaxGroup; ++n) {
+        acc[n] = make_float4(0.f, 0.f, 0.f, 0.f);
+        lsum[n] = 0.f;
+    }
+    for (int rb = r0; rb <= r1; rb += 32) {
+        const int r = rb + lane;
+        float e[kMaxGroup];
+        if (r <= r1) {
+            const float4 *ml = reinterpret_cast<const float4 *>(p.ws_ml + slot_of(r) * kSlotMl);
+#pragma unroll
+            for (int q4 = 0; q4 < kMaxGroup / 2; ++q4) {
+                const float4 v = __ldcg(ml + q4);
+                e[2 * q4] = 2 * q4 < g ? ex2(v.x - M[2 * q4]) : 0.f;
+                e[2 * q4 + 1] = 2 * q4 + 1 < g ? ex2(v.z - M[2 * q4 + 1]) : 0.f;
+                lsum[2 * q4] += e[2 * q4] * v.y;
+                lsum[2 * q4 + 1] += e[2 * q4 + 1] * v.w;
+            }
+        } else {
+#pragma unroll
+            for (int n = 0; n < kMaxGroup; ++n) e[n] = 0.f;
+        }
+        const int cnt = min(32, r1 - rb + 1);
+        for (int i = 0; i < cnt; ++i) {
+            const float *src = p.ws_acc + slot_of(rb + i) * kSlotFloats + 4 * lane;
+            float4 v[kMaxGroup];
+#pragma unroll
+            for (int n = 0; n < kMaxGroup; ++n)
+                if (n < g) v[n] = __ldcg(reinterpret_cast<const float4 *>(src + n * kHeadDim));
+#pragma unroll
+            for (int n = 0; n < kMaxGroup; ++n) {
+                const float en = __shfl_sync(kFull, e[n], i);
+                if (n < g) {
+                    acc[n].x += en * v[n].x; acc[n].y += en * v[n].y;
+                    acc[n].z += en * v[n].z; acc[n].w += en * v[n].w;
+                }
+            }
+        }
+    }
+#pragma unroll
+    for (int n = 0; n < kMaxGroup; ++n)
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) lsum[n] += __shfl_xor_sync(kFull, lsum[n], o);
+    uint16_t *o = p.out + ((size_t)s * p.num_q_heads + (size_t)h * g) * kHeadDim + 4 * lane;
+#pragma unroll
+    for (int n = 0; n < kMaxGroup; ++n) {
+        if (n < g) {
+            const float inv = 1.f / lsum[n];
+            uint16_t *on = o + n * kHeadDim;
+            on[0] = f2bf(acc[n].x * inv); on[1] = f2bf(acc[n].y * inv);
+            on[2] = f2bf(acc[n].z * inv); on[3] = f2bf(acc[n].w * inv);
+        }
+    }
+}
+
+// --------------------------------------------------------------- kernel ----
 
 __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
-    ps_decode_partial_kernel(const PartialParams p, const __grid_constant__ CUtensorMap tmK,
-                             const __grid_constant__ CUtensorMap tmV) {
+    ps_decode_kernel(const DecodeParams p, const __grid_constant__ CUtensorMap tmK,
+                     const __grid_constant__ CUtensorMap tmV) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kWorkersPerCta * kWorkerBytes);
-    int *sP = reinterpret_cast<int *>(bars + kWorkersPerCta * kStages);  // [S + 1] tile prefix (x Hkv)
-    int *sL = sP + p.num_seqs + 1;                                        // [S] clamped lengths
+    int4 *metas = reinterpret_cast<int4 *>(bars + kWorkersPerCta * kStages);  // per stage: pos, range b, e, id
+    int *sP = reinterpret_cast<int *>(metas + kWorkersPerCta * kStages);      // [S + 1] tile prefix (x Hkv)
+    int *sL = sP + p.num_seqs + 1;                                            // [S] clamped lengths
     __shared__ int warp_sums[kWorkersPerCta];
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int S = p.num_seqs, Hkv = p.num_kv_heads, g = p.group, bs = p.block_size;
+    unsigned *status = reinterpret_cast<unsigned *>(p.ws_header + kHdrStatus);
 
-    // 1. Clamped lengths and the exclusive prefix of tiles x kv-heads.
+    // 1. Warm L2 with this CTA's slice of the block table, then build the
+    //    clamped lengths and the exclusive prefix of tiles x kv-heads.
     {
+        const size_t lines = ((size_t)S * p.max_blocks_per_seq * 4 + 127) / 128;
+        for (size_t i = blockIdx.x + (size_t)tid * gridDim.x; i < lines; i += (size_t)blockDim.x * gridDim.x)
+            prefetch_l2(reinterpret_cast<const char *>(p.block_table) + i * 128);
         const int nthr = blockDim.x;
         const int per = (S + nthr - 1) / nthr;
         const int lo = min(S, tid * per), hi = min(S, lo + per);
@@ -227,7 +345,7 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
             sL[i] = L;
             sum += tiles_of(L) * Hkv;
         }
-        if (clamped && blockIdx.x == 0) atomicOr(reinterpret_cast<unsigned *>(p.ws_header + kHdrStatus), kFlagLenClamped);
+        if (clamped && blockIdx.x == 0) atomicOr(status, kFlagLenClamped);
         int incl = sum;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
@@ -248,36 +366,42 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
         fence_mbar_init();
         __syncthreads();
     }
+    // Empty sequences produce zero rows (CTA-strided over sequences).
+    for (int s = blockIdx.x; s < S; s += gridDim.x) {
+        if (sL[s] != 0) continue;
+        uint32_t *o = reinterpret_cast<uint32_t *>(p.out + (size_t)s * p.num_q_heads * kHeadDim);
+        for (int i = tid; i < p.num_q_heads * kHeadDim / 2; i += blockDim.x) o[i] = 0u;
+    }
 
-    const int N = sP[S];
-    long long W = (long long)gridDim.x * kWorkersPerCta;
-    if (p.max_workers > 0 && W > p.max_workers) W = p.max_workers;
+    // 2. Partition of the tape (identical in every CTA).
+    Partition part;
+    const int W = gridDim.x * kWorkersPerCta;
+    part.N = sP[S];
+    const int D = p.dynamic_permille > 0 ? (int)((long long)part.N * p.dynamic_permille / 1000) : 0;
+    part.Ns = part.N - D;
     {
-        const long long cap = (N + p.min_stages - 1) / p.min_stages;
-        if (W > cap) W = cap;
+        int ws = min(W, p.max_workers);
+        const int cap = (part.Ns + p.min_stages - 1) / p.min_stages;
+        part.Ws = part.Ns > 0 ? max(1, min(ws, cap)) : 0;
+        const int per = (D + kChunksPerWorker * W - 1) / (kChunksPerWorker * W);
+        part.Cd = max(kMinChunkTiles, per);
+        part.K = D > 0 ? (D + part.Cd - 1) / part.Cd : 0;
     }
-    if (blockIdx.x == 0) {
-        for (int i = tid; i <= S; i += blockDim.x) p.ws_prefix[i] = sP[i];
-        if (tid == 0) {
-            p.ws_header[kHdrTotalStages] = N;
-            p.ws_header[kHdrWorkers] = (int)W;
-        }
-    }
-    // Worker ids interleave CTAs first so that a small W still spreads over SMs.
-    const int w = warp * gridDim.x + blockIdx.x;
-    if (N == 0 || w >= W) return;
-    const int begin = (int)((long long)w * N / W);
-    const int total = (int)((long long)(w + 1) * N / W) - begin;
-    if (total <= 0) return;
+    const int w = warp * gridDim.x + blockIdx.x;  // CTAs first: a small Ws still spreads over SMs
 
     uint8_t *wbase = smem + warp * kWorkerBytes;
     uint8_t *qslots = wbase + kStages * kStageBytes;
     uint64_t *wbars = bars + warp * kStages;
+    int4 *wmeta = metas + warp * kStages;
     const int mbps = p.max_blocks_per_seq;
 
     // ---- issue side: TMA producer state (lane 0 issues, all lanes track) ----
-    Cursor ic = locate(sP, sL, S, Hkv, begin);
+    int cur_rid = -1, cur_b = 0, cur_e = 0, ip = 0;
+    Cursor ic{0, 0, 0, 0};
     int issued = 0, pieces_issued = 0;
+    bool issue_done = part.N == 0;
+    bool claim_pending = false;
+    int claim_k = 0;                         // valid in lane 0 while a claim is pending
     int win_s = -1, win_j0 = 0, win_v = -1;  // block-table window, one entry per lane
     int pre_s = -1, pre_j0 = 0, pre_v = -1;  // prefetched next window
 
@@ -303,10 +427,30 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
         pre_s = ns_; pre_j0 = nj0;
         pre_v = fetch_window(ns_, nj0);
     };
-
+    auto start_range = [&](int rid) {
+        cur_rid = rid;
+        cur_b = part.range_begin(rid);
+        cur_e = part.range_end(rid);
+        ip = cur_b;
+        ic = locate(sP, sL, S, ip);
+    };
+    auto claim = [&]() {
+        if (lane == 0) claim_k = atomicAdd(p.ws_header + kHdrNextChunk, 1);
+        claim_pending = true;
+    };
+    // Move to the next range: the claimed dynamic chunk, if any.
+    auto next_range = [&]() -> bool {
+        if (part.K == 0) { issue_done = true; return false; }
+        if (!claim_pending) claim();
+        const int k = __shfl_sync(kFull, claim_k, 0);
+        claim_pending = false;
+        if (k >= part.K) { issue_done = true; return false; }
+        start_range(part.Ws + k);
+        return true;
+    };
     auto issue_one = [&]() {
         const int slot = issued % kStages;
-        const bool new_piece = issued == 0 || ic.st == 0;
+        const bool new_piece = ip == cur_b || ic.st == 0;
         const int tok = ic.st * kTileTokens;
         const int j = tok / bs, tok0 = tok - j * bs, j0 = j & ~31;
         if (win_s != ic.s || win_j0 != j0) {
@@ -325,8 +469,9 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
             int row = pb * Hkv + ic.h;
             if (pb < 0 || (long long)pb >= p.num_blocks) {
                 row = -1;  // fully out of bounds: TMA fills zeros
-                atomicOr(reinterpret_cast<unsigned *>(p.ws_header + kHdrStatus), kFlagBadBlock);
+                atomicOr(status, kFlagBadBlock);
             }
+            wmeta[slot] = make_int4(ip, cur_b, cur_e, cur_rid);
             const uint32_t bar = smem_addr(&wbars[slot]);
             const uint32_t dst = smem_addr(wbase + slot * kStageBytes);
             const uint32_t qbytes = new_piece ? (uint32_t)(g * kHeadDim * 2) : 0u;
@@ -343,44 +488,60 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
         }
         if (new_piece) ++pieces_issued;
         ++issued;
-        if (issued < total) advance(ic, sL, S, Hkv);
+        if (++ip < cur_e) advance(ic, sL, S, Hkv);
+        if (part.K > 0 && !claim_pending && cur_e - ip <= kClaimAhead) claim();
     };
 
     // ---- consume side state ----
-    Cursor cc = locate(sP, sL, S, Hkv, begin);
-    int pieces_loaded = 0;
-    bool first_piece = true, piece_from_start = false;
+    Cursor cc{0, 0, 0, 0};
+    int c_rid = 0, c_b = 0, c_e = 0;
+    int pieces_loaded = 0, piece_pos0 = 0;
+    bool piece_from_seg_start = false;
     uint32_t qf[16];
     float acc[8][4];
     float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
 
     auto refill = [&](int consumed) {
-        while (issued < total && issued - consumed < kStages) {
-            const bool np_ = issued == 0 || ic.st == 0;
+        while (!issue_done && issued - consumed < kStages) {
+            if (ip >= cur_e) {
+                if (!next_range()) break;
+                continue;
+            }
+            const bool np_ = ip == cur_b || ic.st == 0;
             if (np_ && pieces_issued >= pieces_loaded + kQSlots) break;
             issue_one();
         }
     };
 
-    refill(0);
+    if (w < part.Ws) start_range(w);
     const int h0 = 2 * (lane & 3), h1 = h0 + 1;
     const int trow = lane >> 2;  // token row of this lane in the S^T fragment
     int consumed = 0;
-    for (; consumed < total;) {
+    refill(0);
+    while (consumed < issued) {
         const int slot = consumed % kStages;
         const bool arrived = mbar_wait(smem_addr(&wbars[slot]), (uint32_t)((consumed / kStages) & 1));
         if (!__all_sync(kFull, arrived)) {
-            if (lane == 0) atomicOr(reinterpret_cast<unsigned *>(p.ws_header + kHdrStatus), kFlagTimeout);
+            if (lane == 0) atomicOr(status, kFlagTimeout);
             // Drain this worker's outstanding copies (bounded) before leaving.
             for (int k = consumed + 1; k < issued; ++k)
                 mbar_wait(smem_addr(&wbars[k % kStages]), (uint32_t)((k / kStages) & 1));
-            return;
+            break;
+        }
+        __syncwarp();
+        const int4 meta = wmeta[slot];
+        const int pos = meta.x;
+        if (pos == meta.y) {
+            cc = locate(sP, sL, S, pos);
+            c_b = meta.y; c_e = meta.z; c_rid = meta.w;
+        } else {
+            advance(cc, sL, S, Hkv);
         }
         const uint8_t *stage = wbase + slot * kStageBytes;
         const uint32_t sK = smem_addr(stage), sV = sK + kTileBytes;
-        const bool piece_start = consumed == 0 || cc.st == 0;
+        const bool piece_start = pos == c_b || cc.st == 0;
         const bool seg_last = cc.st == cc.ns - 1;
-        const bool piece_end = consumed == total - 1 || seg_last;
+        const bool piece_end = pos == c_e - 1 || seg_last;
 
         if (piece_start) {
             const uint32_t qs = smem_addr(qslots + (pieces_loaded % kQSlots) * kQSlotBytes);
@@ -393,7 +554,8 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
                 for (int i = 0; i < 16; ++i) qf[i] = 0u;
             }
             ++pieces_loaded;
-            piece_from_start = cc.st == 0;
+            piece_pos0 = pos;
+            piece_from_seg_start = cc.st == 0;
             m0 = m1 = -INFINITY;
             l0 = l1 = 0.f;
 #pragma unroll
@@ -474,8 +636,8 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
                 L1 += __shfl_xor_sync(kFull, L1, o);
             }
             const int drow = lane >> 2;
-            if (piece_from_start && seg_last) {
-                // The worker saw the whole segment: write the bf16 output rows.
+            if (piece_from_seg_start && seg_last) {
+                // One range covered the whole segment: write the bf16 output rows.
                 uint16_t *o = p.out + ((size_t)cc.s * p.num_q_heads + (size_t)cc.h * g) * kHeadDim;
                 const float i0 = 1.f / L0, i1 = 1.f / L1;
 #pragma unroll
@@ -491,114 +653,72 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
                     }
                 }
             } else {
-                // Cut by a worker boundary: leave (m, l, acc) for the combine.
-                const size_t slotid = 2 * (size_t)w + (first_piece ? 0 : 1);
+                // Cut by a range boundary: leave (m, l, acc) and count the tiles.
+                const size_t slotid = 2 * (size_t)c_rid + (piece_pos0 == c_b ? 0 : 1);
                 float *A = p.ws_acc + slotid * kSlotFloats;
 #pragma unroll
                 for (int mt = 0; mt < 8; ++mt) {
                     const int d = mt * 16 + drow;
-                    A[h0 * kHeadDim + d] = acc[mt][0];
-                    A[h0 * kHeadDim + d + 8] = acc[mt][2];
-                    A[h1 * kHeadDim + d] = acc[mt][1];
-                    A[h1 * kHeadDim + d + 8] = acc[mt][3];
+                    if (h0 < g) {
+                        A[h0 * kHeadDim + d] = acc[mt][0];
+                        A[h0 * kHeadDim + d + 8] = acc[mt][2];
+                    }
+                    if (h1 < g) {
+                        A[h1 * kHeadDim + d] = acc[mt][1];
+                        A[h1 * kHeadDim + d + 8] = acc[mt][3];
+                    }
                 }
                 if (lane < 4) {
                     float *ML = p.ws_ml + slotid * kSlotMl;
                     ML[2 * h0] = m0; ML[2 * h0 + 1] = L0;
                     ML[2 * h1] = m1; ML[2 * h1 + 1] = L1;
                 }
+                __threadfence();
+                __syncwarp();
+                int done = 0;
+                const int tiles = pos - piece_pos0 + 1;
+                int *cnt = p.seg_done + (size_t)cc.s * Hkv + cc.h;
+                if (lane == 0) done = atomicAdd(cnt, tiles) + tiles;
+                done = __shfl_sync(kFull, done, 0);
+                if (done == cc.ns) {
+                    __threadfence();
+                    const int a = sP[cc.s] + cc.h * cc.ns;
+                    merge_segment(p, part, a, a + cc.ns, cc.s, cc.h, lane);
+                    if (lane == 0) *cnt = 0;
+                }
             }
-            first_piece = false;
         }
         ++consumed;
-        if (consumed < total) advance(cc, sL, S, Hkv);
         refill(consumed);
     }
-}
-
-// ------------------------------------------------------ combine kernel ----
-
-__device__ __forceinline__ int worker_of(long long x, long long N, long long W) {
-    return (int)(((x + 1) * W - 1) / N);
-}
-
-constexpr int kCombineWarps = 8;
-
-__global__ void __launch_bounds__(kCombineWarps * 32) ps_decode_combine_kernel(const CombineParams p) {
-    const int s = blockIdx.x;
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int g = p.group;
-    const long long N = p.ws_header[kHdrTotalStages];
-    const long long W = p.ws_header[kHdrWorkers];
-    const int P0 = p.ws_prefix[s], P1 = p.ws_prefix[s + 1];
-    const int ns = (P1 - P0) / p.num_kv_heads;
-    for (int h = warp; h < p.num_kv_heads; h += kCombineWarps) {
-        uint16_t *o = p.out + ((size_t)s * p.num_q_heads + (size_t)h * g) * kHeadDim;
-        if (ns == 0) {
-            for (int i = lane; i < g * kHeadDim; i += 32) o[i] = 0;
-            continue;
-        }
-        const long long a = P0 + (long long)h * ns, b = a + ns;
-        const int wf = worker_of(a, N, W), wl = worker_of(b - 1, N, W);
-        if (wf == wl) continue;  // the partial kernel wrote this segment
-        const long long Rf = (long long)wf * N / W;
-        auto slot_of = [&](int wk) -> size_t {
-            return (wk == wf && Rf != a) ? 2 * (size_t)wk + 1 : 2 * (size_t)wk;
-        };
-        for (int n = 0; n < g; ++n) {
-            float M = -INFINITY;
-            for (int wk = wf + lane; wk <= wl; wk += 32) M = fmaxf(M, p.ws_ml[slot_of(wk) * kSlotMl + 2 * n]);
-#pragma unroll
-            for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(kFull, M, off));
-            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-            float lsum = 0.f;
-            for (int w0 = wf; w0 <= wl; w0 += 32) {
-                const int wk = w0 + lane;
-                float e = 0.f;
-                if (wk <= wl) {
-                    const float *ml = p.ws_ml + slot_of(wk) * kSlotMl + 2 * n;
-                    e = ex2(ml[0] - M);
-                    lsum += e * ml[1];
-                }
-                const int cnt = min(32, wl - w0 + 1);
-                for (int i = 0; i < cnt; ++i) {
-                    const float ei = __shfl_sync(kFull, e, i);
-                    const float4 v = *reinterpret_cast<const float4 *>(p.ws_acc + slot_of(w0 + i) * kSlotFloats +
-                                                                       (size_t)n * kHeadDim + 4 * lane);
-                    acc.x += ei * v.x; acc.y += ei * v.y; acc.z += ei * v.z; acc.w += ei * v.w;
-                }
-            }
-#pragma unroll
-            for (int off = 16; off > 0; off >>= 1) lsum += __shfl_xor_sync(kFull, lsum, off);
-            const float inv = 1.f / lsum;
-            uint16_t *on = o + n * kHeadDim + 4 * lane;
-            on[0] = f2bf(acc.x * inv); on[1] = f2bf(acc.y * inv);
-            on[2] = f2bf(acc.z * inv); on[3] = f2bf(acc.w * inv);
+    // The last warp to finish resets the chunk dispenser for the next call.
+    if (lane == 0) {
+        __threadfence();
+        const int n = atomicAdd(p.ws_header + kHdrWarpsDone, 1);
+        if (n == W - 1) {
+            p.ws_header[kHdrNextChunk] = 0;
+            p.ws_header[kHdrWarpsDone] = 0;
+            __threadfence();
         }
     }
 }
 
 }  // namespace
 
-cudaError_t launch_partial(const PartialParams &p, const CUtensorMap &tmK, const CUtensorMap &tmV, int grid_ctas,
-                           size_t smem_bytes, cudaStream_t stream) {
+cudaError_t launch_decode(const DecodeParams &p, const CUtensorMap &tmK, const CUtensorMap &tmV, int grid_ctas,
+                          size_t smem_bytes, cudaStream_t stream) {
     static bool attr_done[64] = {};
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
     if (!attr_done[dev]) {
-        e = cudaFuncSetAttribute(ps_decode_partial_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        e = cudaFuncSetAttribute(ps_decode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)partial_smem_bytes(kMaxSeqs));
         if (e != cudaSuccess) return e;
         attr_done[dev] = true;
     }
-    ps_decode_partial_kernel<<<grid_ctas, kWorkersPerCta * 32, smem_bytes, stream>>>(p, tmK, tmV);
-    return cudaGetLastError();
-}
-
-cudaError_t launch_combine(const CombineParams &p, cudaStream_t stream) {
-    ps_decode_combine_kernel<<<p.num_seqs, kCombineWarps * 32, 0, stream>>>(p);
+    ps_decode_kernel<<<grid_ctas, kWorkersPerCta * 32, smem_bytes, stream>>>(p, tmK, tmV);
     return cudaGetLastError();
 }
 

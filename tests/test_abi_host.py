@@ -37,7 +37,7 @@ def test_status_strings_and_version():
 
 def _plan(**kw):
     args = dict(num_seqs=64, num_q_heads=32, num_kv_heads=8, head_dim=128, block_size=16, max_blocks_per_seq=256,
-                num_blocks=12000, num_sms=152, max_workers=0, min_stages_per_worker=0)
+                num_blocks=12000, num_sms=152, max_workers=0, min_stages_per_worker=0, dynamic_permille=-1)
     args.update(kw)
     return psd.ps_decode_plan_create_ex(**args)
 
@@ -47,11 +47,13 @@ def test_plan_sizing_matches_layout():
     try:
         info = psd.ps_decode_plan_info(plan)
         assert info["grid_ctas"] == 152
-        assert info["workers_per_cta"] == 4
-        W = 152 * 4
+        W = 152 * info["workers_per_cta"]
         assert info["max_workers"] == W
-        # header + prefix (S + 1 ints) + 2W partial slots of 8 heads x (128 acc + m, l) fp32
-        expect = 256 + 512 + 2 * W * 8 * 128 * 4 + 2 * W * 8 * 2 * 4
+        assert info["dynamic_permille"] == 0
+        # header + per-segment counters (S x Hkv ints) + partial slots: two per static range
+        # and per dynamic chunk (at most 4 per worker), 8 heads x (128 acc + m, l) fp32 each
+        slots = 2 * W * 5
+        expect = 256 + 64 * 8 * 4 + slots * 8 * 128 * 4 + slots * 8 * 2 * 4
         assert ws == info["workspace_bytes"]
         assert expect <= ws <= expect + 3 * 256
         assert info["smem_bytes"] <= 227 * 1024
@@ -77,6 +79,8 @@ def test_max_seqs_plan_fits_shared_memory():
     (dict(num_seqs=4097), psd.PS_ERR_UNSUPPORTED),
     (dict(num_blocks=0), psd.PS_ERR_INVALID_ARG),
     (dict(num_sms=-1), psd.PS_ERR_INVALID_ARG),
+    (dict(dynamic_permille=1001), psd.PS_ERR_INVALID_ARG),
+    (dict(dynamic_permille=-2), psd.PS_ERR_INVALID_ARG),
 ])
 def test_plan_rejects_bad_shapes(kw, status):
     with pytest.raises(psd.PsError) as ei:
@@ -143,9 +147,10 @@ def test_stream_binding_lookup():
 
 
 def test_worker_overrides_are_recorded():
-    plan, _ = _plan(max_workers=1, min_stages_per_worker=3)
+    plan, _ = _plan(max_workers=1, min_stages_per_worker=3, dynamic_permille=0)
     try:
         info = psd.ps_decode_plan_info(plan)
         assert info["max_workers"] == 1 and info["min_stages_per_worker"] == 3
+        assert info["dynamic_permille"] == 0
     finally:
         psd.ps_decode_plan_destroy(plan)
