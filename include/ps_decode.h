@@ -187,6 +187,46 @@ ps_status_t ps_decode_plan_set_timing_events(ps_decode_plan_t *plan, void *ev_st
 ps_status_t ps_decode_plan_read_device_status(ps_decode_plan_t *plan, void *stream,
                                               unsigned int *flags);
 
+/*
+ * Decode attention for callers that cannot allocate device memory.  (The
+ * paper has no counterpart; this is a deployment convenience.)
+ *
+ * Some callers can pass the library their tensors but cannot give it a
+ * workspace: plugins whose host engine owns every device allocation, callers
+ * over a foreign-function interface that hold only the buffers they pass in,
+ * or serving processes that budget all device memory at start-up and forbid
+ * allocations afterwards.  This entry point needs no plan and no workspace:
+ * the split-KV scratch lives in a fixed device array inside the library of
+ * PS_NOALLOC_SCRATCH_BYTES, which every GPU that loads the library holds
+ * until the process exits.  It calls no cudaMalloc, cudaFree or other
+ * allocating routine.
+ *
+ * Arguments are those of ps_decode_attention() plus the two a plan would
+ * otherwise supply: max_blocks_per_seq (the block_table row stride) and
+ * num_blocks (physical blocks in k_cache / v_cache).  The work is split
+ * statically, with the same kernel and the same numerics as the planned path.
+ *
+ * - The first call on each device resolves the device address of the scratch
+ *   array (and sets the kernel's shared-memory limit) on that device; make
+ *   that first call before any stream capture.
+ * - Every call shares the one array and first clears its counters on
+ *   `stream`.  Calls that overlap on the GPU (other streams, other host
+ *   threads) race on the array and produce wrong results: serialise them.
+ * - Shapes whose scratch need exceeds PS_NOALLOC_SCRATCH_BYTES (2 partial
+ *   states of 8 x 130 floats per streaming warp, plus 4 bytes per
+ *   (sequence, kv-head)) return PS_ERR_UNSUPPORTED before anything is
+ *   launched.
+ * - Launches through this entry point are not counted by
+ *   ps_decode_launch_count(), and there is no device status word to read.
+ * Errors: PS_ERR_INVALID_ARG, PS_ERR_UNSUPPORTED, PS_ERR_CUDA.
+ */
+#define PS_NOALLOC_SCRATCH_BYTES (16u << 20)
+ps_status_t ps_decode_attention_noalloc(const void *q, const void *k_cache, const void *v_cache,
+                                        const int *block_table, const int *seq_lens, void *out,
+                                        int num_seqs, int num_q_heads, int num_kv_heads, int head_dim,
+                                        int block_size, int max_blocks_per_seq, long long num_blocks,
+                                        float scale, void *stream);
+
 /* Number of kernels this library has launched in this process. */
 unsigned long long ps_decode_launch_count(void);
 

@@ -1,0 +1,167 @@
+// ps_decode_noalloc.cu -- decode attention for callers that cannot allocate.
+//
+// Some callers have no way to hand the library a workspace: a host engine
+// whose device memory is owned by an allocator the plugin may not call,
+// a foreign-function caller that only holds the tensors it passes in, or a
+// serving process that accounts every byte up front and forbids any
+// allocation after start-up.  ps_decode_attention_noalloc() serves them.  It
+// runs the same kernel as ps_decode_attention_planned() with a fully static
+// split, and keeps the split-KV scratch (counters and partial softmax
+// states) in the fixed device array below instead of a caller workspace.
+// Nothing here calls cudaMalloc, cudaFree or any allocating routine.
+//
+// The array costs every GPU that loads the library kNoallocScratchBytes of
+// device memory until the process exits.  All calls share it, and it keeps
+// whatever the previous call left there, so each call first clears the part
+// that must start at zero; two calls that overlap on the GPU (different
+// streams, or different host threads) race on it and give wrong results.
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdint>
+#include <mutex>
+
+#include "ps_decode.h"
+#include "ps_internal.h"
+
+namespace {
+
+constexpr size_t kNoallocScratchBytes = (size_t)PS_NOALLOC_SCRATCH_BYTES;
+
+// The scratch itself.  Host code must not use this name as an address: it is
+// a host-side stand-in for the device symbol.  The device address comes from
+// cudaGetSymbolAddress() below.
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoallocScratchBytes];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_setup_mu;
+void *g_scratch_ptr[kMaxDevices] = {};
+
+// Device address of the scratch array on the current device, resolved once per
+// device (with that device current) on the first call made on it.
+cudaError_t scratch_address(void **out) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lk(g_setup_mu);
+    if (g_scratch_ptr[dev] == nullptr) {
+        void *ptr = nullptr;
+        e = cudaGetSymbolAddress(&ptr, g_noalloc_scratch);
+        if (e != cudaSuccess) return e;
+        g_scratch_ptr[dev] = ptr;
+    }
+    *out = g_scratch_ptr[dev];
+    return cudaSuccess;
+}
+
+using EncodeTiledFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                   const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn tiled_encoder() {
+    static EncodeTiledFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *f = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(f);
+    });
+    return fn;
+}
+
+// Same 3-D view of a paged cache the planned path uses: dims (head_dim, slot,
+// block x kv-head), box 64 x 16 x 1, 128-byte swizzle.
+bool encode_cache(CUtensorMap *tm, const void *base, int block_size, long long num_blocks, int num_kv_heads) {
+    EncodeTiledFn fn = tiled_encoder();
+    if (!fn) return false;
+    cuuint64_t dims[3] = {(cuuint64_t)ps::kHeadDim, (cuuint64_t)block_size,
+                          (cuuint64_t)num_blocks * (cuuint64_t)num_kv_heads};
+    cuuint64_t strides[2] = {(cuuint64_t)ps::kHeadDim * 2, (cuuint64_t)block_size * ps::kHeadDim * 2};
+    cuuint32_t box[3] = {64, (cuuint32_t)ps::kTileTokens, 1};
+    cuuint32_t estr[3] = {1, 1, 1};
+    return fn(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool is_aligned(const void *p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
+
+}  // namespace
+
+extern "C" ps_status_t ps_decode_attention_noalloc(const void *q, const void *k_cache, const void *v_cache,
+                                                   const int *block_table, const int *seq_lens, void *out,
+                                                   int num_seqs, int num_q_heads, int num_kv_heads, int head_dim,
+                                                   int block_size, int max_blocks_per_seq, long long num_blocks,
+                                                   float scale, void *stream) {
+    using namespace ps;
+    if (!q || !k_cache || !v_cache || !block_table || !seq_lens || !out) return PS_ERR_INVALID_ARG;
+    if (!is_aligned(q, 16) || !is_aligned(k_cache, 16) || !is_aligned(v_cache, 16) || !is_aligned(out, 16) ||
+        !is_aligned(block_table, 4) || !is_aligned(seq_lens, 4))
+        return PS_ERR_INVALID_ARG;
+    if (num_seqs <= 0 || num_q_heads <= 0 || num_kv_heads <= 0 || head_dim <= 0 || block_size <= 0 ||
+        max_blocks_per_seq <= 0 || num_blocks <= 0 || num_q_heads % num_kv_heads != 0 || !std::isfinite(scale))
+        return PS_ERR_INVALID_ARG;
+    if (head_dim != kHeadDim || num_q_heads / num_kv_heads > kMaxGroup || block_size % kTileTokens != 0 ||
+        block_size > 256 || num_seqs > kMaxSeqs)
+        return PS_ERR_UNSUPPORTED;
+    const long long len_cap = (long long)max_blocks_per_seq * block_size;
+    if (len_cap > INT32_MAX || (long long)num_seqs * ((len_cap + kTileTokens - 1) / kTileTokens) * num_kv_heads > INT32_MAX ||
+        num_blocks * num_kv_heads > INT32_MAX)
+        return PS_ERR_UNSUPPORTED;
+
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0)
+        return PS_ERR_CUDA;
+    // Scratch layout: header, per-segment counters, then two partial slots per
+    // static worker range (no dynamic chunks on this path).
+    const int workers = sms * kWorkersPerCta;
+    const size_t seg_off = kWsHeaderBytes;
+    const size_t acc_off = align_up(seg_off + (size_t)num_seqs * num_kv_heads * 4, 256);
+    const size_t slots = 2 * (size_t)workers;
+    const size_t ml_off = align_up(acc_off + slots * kSlotFloats * 4, 256);
+    const size_t need = align_up(ml_off + slots * kSlotMl * 4, 256);
+    if (need > kNoallocScratchBytes) return PS_ERR_UNSUPPORTED;  // beyond the fixed scratch array
+
+    void *scratch = nullptr;
+    if (scratch_address(&scratch) != cudaSuccess) return PS_ERR_CUDA;
+    CUtensorMap tmK, tmV;
+    if (!encode_cache(&tmK, k_cache, block_size, num_blocks, num_kv_heads) ||
+        !encode_cache(&tmV, v_cache, block_size, num_blocks, num_kv_heads))
+        return PS_ERR_CUDA;
+
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    uint8_t *ws = static_cast<uint8_t *>(scratch);
+    // Counters and the status word must start at zero; the previous call's
+    // contents are still in the array.
+    if (cudaMemsetAsync(ws, 0, acc_off, st) != cudaSuccess) return PS_ERR_CUDA;
+
+    DecodeParams dp;
+    dp.q = static_cast<const uint16_t *>(q);
+    dp.block_table = block_table;
+    dp.seq_lens = seq_lens;
+    dp.out = static_cast<uint16_t *>(out);
+    dp.ws_header = reinterpret_cast<int *>(ws);
+    dp.seg_done = reinterpret_cast<int *>(ws + seg_off);
+    dp.ws_acc = reinterpret_cast<float *>(ws + acc_off);
+    dp.ws_ml = reinterpret_cast<float *>(ws + ml_off);
+    dp.num_seqs = num_seqs;
+    dp.num_q_heads = num_q_heads;
+    dp.num_kv_heads = num_kv_heads;
+    dp.group = num_q_heads / num_kv_heads;
+    dp.block_size = block_size;
+    dp.max_blocks_per_seq = max_blocks_per_seq;
+    dp.num_blocks = num_blocks;
+    dp.len_cap = (int)len_cap;
+    dp.max_workers = workers;
+    dp.min_stages = kDefaultMinStages;
+    dp.dynamic_permille = 0;
+    dp.scale_log2 = (float)((double)scale * 1.4426950408889634);
+    if (launch_decode(dp, tmK, tmV, sms, partial_smem_bytes(num_seqs), st) != cudaSuccess) return PS_ERR_CUDA;
+    return PS_OK;
+}

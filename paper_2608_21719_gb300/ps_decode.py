@@ -72,6 +72,8 @@ _SIGS = {
     "ps_decode_attention_planned": (_i, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _f, _vp]),
     "ps_decode_plan_set_timing_events": (_i, [_vp, _vp, _vp]),
     "ps_decode_plan_read_device_status": (_i, [_vp, _vp, ctypes.POINTER(ctypes.c_uint)]),
+    "ps_decode_attention_noalloc": (_i, [_vp, _vp, _vp, _vp, _vp, _vp, _i, _i, _i, _i, _i, _i, ctypes.c_longlong,
+                                         _f, _vp]),
     "ps_decode_launch_count": (ctypes.c_ulonglong, []),
     "ps_status_string": (ctypes.c_char_p, [_i]),
     "ps_decode_abi_version": (_i, []),
@@ -171,6 +173,17 @@ def ps_decode_attention_planned(plan, q, k_cache, v_cache, block_table, seq_lens
     _check(_lib.ps_decode_attention_planned(plan, _ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(block_table),
                                             _ptr(seq_lens), _ptr(out), float(scale), _stream(stream)),
            "ps_decode_attention_planned")
+
+
+def ps_decode_attention_noalloc(q, k_cache, v_cache, block_table, seq_lens, out, num_seqs, num_q_heads,
+                                num_kv_heads, head_dim, block_size, max_blocks_per_seq, num_blocks, scale,
+                                stream) -> None:
+    """Decode attention with no plan and no workspace (scratch in a fixed
+    device array inside the library; see include/ps_decode.h)."""
+    _check(_lib.ps_decode_attention_noalloc(_ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(block_table),
+                                            _ptr(seq_lens), _ptr(out), num_seqs, num_q_heads, num_kv_heads,
+                                            head_dim, block_size, max_blocks_per_seq, num_blocks, float(scale),
+                                            _stream(stream)), "ps_decode_attention_noalloc")
 
 
 def ps_decode_plan_set_timing_events(plan, ev_start, ev_end) -> None:
