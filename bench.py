@@ -52,6 +52,12 @@ def parse_args(argv=None):
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="CPU time budget of the oracle baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--flush", choices=["write-read", "write"], default="write-read",
+                    help="L2 flush between steps: write a 2x-L2 buffer, then read it back so that "
+                         "L2 holds clean lines (default), or only write it (leaves dirty lines whose "
+                         "write-back lands inside the next timed step)")
+    ap.add_argument("--dynamic-permille", type=int, default=-1,
+                    help="share of the KV stream shared between warps at run time (-1: library default)")
     return ap.parse_args(argv)
 
 
@@ -245,11 +251,24 @@ def run_ours(args):
     lens = wl.seq_lens.cpu().numpy()
     alg = roofline.algorithmic_bytes(lens, wl.num_q_heads, wl.num_kv_heads, wl.head_dim, wl.block_size)
 
-    attn = ps_decode.DecodeAttention.for_workload(wl)
+    attn = ps_decode.DecodeAttention.for_workload(wl, dynamic_permille=args.dynamic_permille)
     out = torch.empty_like(wl.q)
     stream = torch.cuda.current_stream(dev)
     l2 = torch.cuda.get_device_properties(dev).L2_cache_size
-    flush = torch.empty(max(2 * l2, 64 << 20), dtype=torch.uint8, device=dev)
+    flush_buf = torch.empty(max(2 * l2, 64 << 20) // 4, dtype=torch.int32, device=dev)
+    flush_sink = torch.empty((), dtype=torch.int32, device=dev)
+
+    class _Flush:
+        """Evict the inputs from L2 between steps, outside the timed interval."""
+        nbytes = flush_buf.numel() * 4
+
+        @staticmethod
+        def zero_():
+            flush_buf.zero_()
+            if args.flush == "write-read":
+                torch.amax(flush_buf, dim=0, out=flush_sink)
+
+    flush = _Flush
 
     def step():
         attn(wl.q, wl.k_cache, wl.v_cache, wl.block_table, wl.seq_lens, out=out, scale=wl.scale, stream=stream)
@@ -340,7 +359,8 @@ def run_ours(args):
             "head_dim": wl.head_dim, "block_size": wl.block_size, "lengths": list(cfg.lengths),
             "seed": cfg.seed, "total_tokens": int(lens.sum()), "kv_bytes": alg["kv"],
             "pool_blocks": wl.num_blocks,
-            "l2": "flushed before every step (write of %d MB, outside the timed interval)" % (flush.numel() >> 20),
+            "l2": "flushed before every step, outside the timed interval: %s of a %d MB buffer" % (
+                "write then read" if args.flush == "write-read" else "write", flush.nbytes >> 20),
             "parallelism": "replicas" if world == 1 else "dp%d (independent batches per GPU)" % world,
         },
         "frac_of_hbm_peak": round(alg["total"] / (ms_per_step * 1e-3) / 1e9 / hbm_peak, 4),

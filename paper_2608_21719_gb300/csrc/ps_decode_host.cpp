@@ -26,6 +26,7 @@ struct ps_decode_plan {
     void *workspace = nullptr;
     size_t workspace_size = 0;
     bool status_needs_clear = false;
+    unsigned epoch = 0;  // calls since the workspace was last zeroed; tags the dynamic state
     // TMA descriptors for the last (k_cache, v_cache) pair seen.
     const void *tm_k_ptr = nullptr, *tm_v_ptr = nullptr;
     alignas(64) CUtensorMap tmK;
@@ -118,7 +119,9 @@ ps_status_t run_planned(ps_decode_plan *p, const void *q, const void *k, const v
         p->tm_v_ptr = v;
     }
     uint8_t *ws = static_cast<uint8_t *>(p->workspace);
+    if (++p->epoch >= (1u << kEpochBits)) p->status_needs_clear = true;  // epoch wrapped: re-zero the workspace
     if (p->status_needs_clear) {
+        p->epoch = 1;
         // Status word, chunk dispenser and per-segment counters start at zero;
         // the kernel returns them to zero at the end of every call.
         if (cudaMemsetAsync(ws, 0, p->ws.acc_off, st) != cudaSuccess) return PS_ERR_CUDA;
@@ -132,6 +135,8 @@ ps_status_t run_planned(ps_decode_plan *p, const void *q, const void *k, const v
     dp.out = static_cast<uint16_t *>(out);
     dp.ws_header = reinterpret_cast<int *>(ws);
     dp.seg_done = reinterpret_cast<int *>(ws + p->ws.seg_done_off);
+    dp.dyn = reinterpret_cast<unsigned long long *>(ws + p->ws.dyn_off);
+    dp.epoch = p->epoch;
     dp.ws_acc = reinterpret_cast<float *>(ws + p->ws.acc_off);
     dp.ws_ml = reinterpret_cast<float *>(ws + p->ws.ml_off);
     dp.num_seqs = p->num_seqs;

@@ -207,40 +207,86 @@ __device__ __forceinline__ void advance(Cursor &c, const int *sL, int S, int Hkv
     c.ns = c.s < S ? tiles_of(sL[c.s]) : 0;
 }
 
-// Split of the tape into static worker ranges followed by dynamic chunks.
-// Range ids: static ranges 0 .. Ws-1, dynamic chunks Ws .. Ws+K-1, in tape order.
+// Split of the tape: static worker ranges over [0, Ns), then the dynamic
+// segments [Js, S*Hkv) (Ns is a segment start), shared at run time.
 struct Partition {
-    int N, Ns, Ws, Cd, K;
+    int N, Ns, Ws, D, Js;
 
-    __device__ int range_of(int x) const {
-        if (x < Ns) return (int)((((long long)x + 1) * Ws - 1) / Ns);
-        return Ws + (x - Ns) / Cd;
-    }
-    __device__ int range_begin(int r) const {
-        if (r < Ws) return (int)((long long)r * Ns / Ws);
-        return Ns + (r - Ws) * Cd;
-    }
-    __device__ int range_end(int r) const {
-        if (r < Ws) return (int)((long long)(r + 1) * Ns / Ws);
-        return min(N, Ns + (r - Ws + 1) * Cd);
-    }
+    __device__ int range_of(int x) const { return (int)((((long long)x + 1) * Ws - 1) / Ns); }
+    __device__ int range_begin(int r) const { return (int)((long long)r * Ns / Ws); }
+    __device__ int range_end(int r) const { return (int)((long long)(r + 1) * Ns / Ws); }
 };
 
-// Merge every cut piece of segment (s, h) in tape order into bf16 output rows.
-// Pieces are read through L2 (other SMs wrote them).  Lanes take one piece
-// each for the (m, l) pass; for the weighted sum every lane owns dims
-// [4*lane, 4*lane+4) of every head, so all loads of a piece are in flight
-// together.
-__device__ void merge_segment(const DecodeParams &p, const Partition &part, int a, int b, int s, int h, int lane) {
+// Packed per-segment word: [epoch:20 | participants:12 | tile cursor:32].
+constexpr int kEpochShift = 64 - (int)kEpochBits;
+constexpr unsigned long long kJoinInc = 1ull << 32;
+
+// Add `inc` to a packed word and return its previous (participants, cursor)
+// part as seen in this call's epoch; a word still tagged with an older epoch
+// counts as zero.  Returns ~0 if the word could not be brought to the current
+// epoch within a bounded number of attempts.
+__device__ unsigned long long epoch_add(unsigned long long *w, unsigned long long inc, unsigned epoch) {
+    constexpr unsigned long long kValMask = (1ull << kEpochShift) - 1;
+    const unsigned long long tag = (unsigned long long)epoch << kEpochShift;
+    unsigned long long v = atomicAdd(w, inc);
+    if ((v & ~kValMask) == tag) return v & kValMask;
+    unsigned long long cur = v + inc;
+    for (int i = 0; i < 64; ++i) {
+        const unsigned long long prev = atomicCAS(w, cur, tag | inc);
+        if (prev == cur) return 0ull;
+        if ((prev & ~kValMask) == tag) {
+            v = atomicAdd(w, inc);
+            if ((v & ~kValMask) == tag) return v & kValMask;
+            cur = v + inc;
+        } else {
+            cur = prev;
+        }
+    }
+    return ~0ull;
+}
+
+// Join a shared segment and claim its next `claim` tiles in one step, but
+// only while it has fewer than `cap` participants and unclaimed tiles left
+// (a join past the cap must not take tiles it could not register).  Returns
+// the previous (participants, cursor) part, or ~0 if the segment is full,
+// exhausted, or kept changing for a bounded number of attempts.
+__device__ unsigned long long epoch_join(unsigned long long *w, unsigned claim, int cap, int ns, unsigned epoch) {
+    constexpr unsigned long long kValMask = (1ull << kEpochShift) - 1;
+    const unsigned long long tag = (unsigned long long)epoch << kEpochShift;
+    unsigned long long cur = __ldcg(w);
+    for (int i = 0; i < 64; ++i) {
+        const unsigned long long val = (cur & ~kValMask) == tag ? (cur & kValMask) : 0ull;
+        if ((int)(val >> 32) >= cap || (int)(unsigned)val >= ns) return ~0ull;
+        const unsigned long long prev = atomicCAS(w, cur, tag | (val + kJoinInc + claim));
+        if (prev == cur) return val;
+        cur = prev;
+    }
+    return ~0ull;
+}
+
+// (participants, cursor) part of a packed word in this call's epoch (0 if older).
+__device__ __forceinline__ unsigned long long epoch_peek(const unsigned long long *w, unsigned epoch) {
+    constexpr unsigned long long kValMask = (1ull << kEpochShift) - 1;
+    const unsigned long long v = __ldcg(w);
+    return (v >> kEpochShift) == epoch ? (v & kValMask) : 0ull;
+}
+
+// Merge `count` cut pieces of segment (s, h) into bf16 output rows by the
+// log-sum-exp rule.  Piece i's workspace slot comes from slot_lane(i), called
+// only by the lane that owns piece i (i = lane + 32k, may diverge), or from
+// slot_all(i), called by all lanes together with the same i.  Pieces are read
+// through L2 (other SMs wrote them).  Lanes take one piece each for the
+// (m, l) pass; for the weighted sums every lane owns dims [4*lane, 4*lane+4)
+// of every head, so all loads of a piece are in flight together.
+template <typename SlotLane, typename SlotAll>
+__device__ void merge_pieces(const DecodeParams &p, int count, SlotLane slot_lane, SlotAll slot_all, int s, int h,
+                             int lane) {
     const int g = p.group;
-    const int r0 = part.range_of(a), r1 = part.range_of(b - 1);
-    auto slot_of = [&](int r) -> size_t { return 2 * (size_t)r + (part.range_begin(r) < a ? 1 : 0); };
-    // Pass 1: per-head maximum over all pieces of their running maxima.
     float M[kMaxGroup];
 #pragma unroll
     for (int n = 0; n < kMaxGroup; ++n) M[n] = -INFINITY;
-    for (int r = r0 + lane; r <= r1; r += 32) {
-        const float4 *ml = reinterpret_cast<const float4 *>(p.ws_ml + slot_of(r) * kSlotMl);
+    for (int i = lane; i < count; i += 32) {
+        const float4 *ml = reinterpret_cast<const float4 *>(p.ws_ml + slot_lane(i) * kSlotMl);
 #pragma unroll
         for (int q4 = 0; q4 < kMaxGroup / 2; ++q4) {
             const float4 v = __ldcg(ml + q4);
@@ -252,7 +298,6 @@ __device__ void merge_segment(const DecodeParams &p, const Partition &part, int 
     for (int n = 0; n < kMaxGroup; ++n)
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) M[n] = fmaxf(M[n], __shfl_xor_sync(kFull, M[n], o));
-    // Pass 2: weights per piece and head, weighted sums of the pieces.
     float4 acc[kMaxGroup];
     float lsum[kMaxGroup];
 #pragma unroll
@@ -260,11 +305,10 @@ __device__ void merge_segment(const DecodeParams &p, const Partition &part, int 
         acc[n] = make_float4(0.f, 0.f, 0.f, 0.f);
         lsum[n] = 0.f;
     }
-    for (int rb = r0; rb <= r1; rb += 32) {
-        const int r = rb + lane;
+    for (int ib = 0; ib < count; ib += 32) {
         float e[kMaxGroup];
-        if (r <= r1) {
-            const float4 *ml = reinterpret_cast<const float4 *>(p.ws_ml + slot_of(r) * kSlotMl);
+        if (ib + lane < count) {
+            const float4 *ml = reinterpret_cast<const float4 *>(p.ws_ml + slot_lane(ib + lane) * kSlotMl);
 #pragma unroll
             for (int q4 = 0; q4 < kMaxGroup / 2; ++q4) {
                 const float4 v = __ldcg(ml + q4);
@@ -277,9 +321,9 @@ __device__ void merge_segment(const DecodeParams &p, const Partition &part, int 
 #pragma unroll
             for (int n = 0; n < kMaxGroup; ++n) e[n] = 0.f;
         }
-        const int cnt = min(32, r1 - rb + 1);
+        const int cnt = min(32, count - ib);
         for (int i = 0; i < cnt; ++i) {
-            const float *src = p.ws_acc + slot_of(rb + i) * kSlotFloats + 4 * lane;
+            const float *src = p.ws_acc + slot_all(ib + i) * kSlotFloats + 4 * lane;
             float4 v[kMaxGroup];
 #pragma unroll
             for (int n = 0; n < kMaxGroup; ++n)
@@ -318,8 +362,9 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kWorkersPerCta * kWorkerBytes);
-    int4 *metas = reinterpret_cast<int4 *>(bars + kWorkersPerCta * kStages);  // per stage: pos, range b, e, id
-    int *sP = reinterpret_cast<int *>(metas + kWorkersPerCta * kStages);      // [S + 1] tile prefix (x Hkv)
+    int4 *metas = reinterpret_cast<int4 *>(bars + kWorkersPerCta * kStages);  // per stage: tile, piece
+    int4 *pieces = metas + kWorkersPerCta * kStages;                          // per warp: ring of 4 pieces
+    int *sP = reinterpret_cast<int *>(pieces + kWorkersPerCta * 4);           // [S + 1] tile prefix (x Hkv)
     int *sL = sP + p.num_seqs + 1;                                            // [S] clamped lengths
     __shared__ int warp_sums[kWorkersPerCta];
 
@@ -376,16 +421,21 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
     // 2. Partition of the tape (identical in every CTA).
     Partition part;
     const int W = gridDim.x * kWorkersPerCta;
+    const int nseg = S * Hkv;
     part.N = sP[S];
-    const int D = p.dynamic_permille > 0 ? (int)((long long)part.N * p.dynamic_permille / 1000) : 0;
-    part.Ns = part.N - D;
     {
-        int ws = min(W, p.max_workers);
+        const int dnom = p.dynamic_permille > 0 ? (int)((long long)part.N * p.dynamic_permille / 1000) : 0;
+        if (dnom > 0) {
+            const Cursor c = locate(sP, sL, S, part.N - dnom);  // round the split down to a segment start
+            part.Ns = sP[c.s] + c.h * c.ns;
+            part.Js = c.s * Hkv + c.h;
+        } else {
+            part.Ns = part.N;
+            part.Js = nseg;
+        }
+        part.D = part.N - part.Ns;
         const int cap = (part.Ns + p.min_stages - 1) / p.min_stages;
-        part.Ws = part.Ns > 0 ? max(1, min(ws, cap)) : 0;
-        const int per = (D + kChunksPerWorker * W - 1) / (kChunksPerWorker * W);
-        part.Cd = max(kMinChunkTiles, per);
-        part.K = D > 0 ? (D + part.Cd - 1) / part.Cd : 0;
+        part.Ws = part.Ns > 0 ? max(1, min(min(W, p.max_workers), cap)) : 0;
     }
     const int w = warp * gridDim.x + blockIdx.x;  // CTAs first: a small Ws still spreads over SMs
 
@@ -393,33 +443,53 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
     uint8_t *qslots = wbase + kStages * kStageBytes;
     uint64_t *wbars = bars + warp * kStages;
     int4 *wmeta = metas + warp * kStages;
+    int4 *wpieces = pieces + warp * 4;
     const int mbps = p.max_blocks_per_seq;
+    const unsigned epoch = p.epoch;
 
     // ---- issue side: TMA producer state (lane 0 issues, all lanes track) ----
+    // mode 0: static range, 1: dynamic segments, 2: nothing left to issue.
+    int mode = (w < part.Ws) ? 0 : (part.D > 0 ? 1 : 2);
     int cur_rid = -1, cur_b = 0, cur_e = 0, ip = 0;
     Cursor ic{0, 0, 0, 0};
+    if (mode == 0) {
+        cur_rid = w;
+        cur_b = part.range_begin(w);
+        cur_e = part.range_end(w);
+        ip = cur_b;
+        ic = locate(sP, sL, S, ip);
+        if (cur_b >= cur_e) mode = part.D > 0 ? 1 : 2;
+    }
+    // dynamic-phase state
+    int dj = -1, d_s = 0, d_h = 0, d_ns = 0, d_t = 0, d_te = 0, d_reg = 0, d_k = 0, d_kcur = 0;
+    bool d_new = false, la_pending = false;
+    unsigned long long la_val = 0;  // lane 0: result of the claim fired ahead
+    int scan_j = part.Js + (int)((long long)w * (nseg - part.Js) / max(W, 1));
+    int scan_left = nseg - part.Js;
+
     int issued = 0, pieces_issued = 0;
-    bool issue_done = part.N == 0;
-    bool claim_pending = false;
-    int claim_k = 0;                         // valid in lane 0 while a claim is pending
     int win_s = -1, win_j0 = 0, win_v = -1;  // block-table window, one entry per lane
     int pre_s = -1, pre_j0 = 0, pre_v = -1;  // prefetched next window
+    // next tile to issue
+    int nx_s = 0, nx_h = 0, nx_st = 0;
+    bool nx_new = false, have_next = false;
+    int4 nx_piece = make_int4(0, 0, 0, 0);
 
     auto fetch_window = [&](int s, int j0) -> int {
         const int j = j0 + lane;
         const int np = (sL[s] + bs - 1) / bs;
         return j < np ? __ldg(p.block_table + (size_t)s * mbps + j) : -1;
     };
-    // Start loading the window the issue cursor will need after the current one.
-    auto prefetch_next = [&]() {
+    // Start loading the window that will most likely be needed after the current one.
+    auto prefetch_next = [&](int s, int h) {
         int ns_ = -1, nj0 = 0;
-        const int np = (sL[ic.s] + bs - 1) / bs;
+        const int np = (sL[s] + bs - 1) / bs;
         if (win_j0 + 32 < np) {
-            ns_ = ic.s; nj0 = win_j0 + 32;
-        } else if (ic.h + 1 < Hkv) {
-            ns_ = ic.s; nj0 = 0;
+            ns_ = s; nj0 = win_j0 + 32;
+        } else if (h + 1 < Hkv) {
+            ns_ = s; nj0 = 0;
         } else {
-            int s2 = ic.s + 1;
+            int s2 = s + 1;
             while (s2 < S && sL[s2] == 0) ++s2;
             if (s2 < S) { ns_ = s2; nj0 = 0; }
         }
@@ -427,95 +497,269 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
         pre_s = ns_; pre_j0 = nj0;
         pre_v = fetch_window(ns_, nj0);
     };
-    auto start_range = [&](int rid) {
-        cur_rid = rid;
-        cur_b = part.range_begin(rid);
-        cur_e = part.range_end(rid);
-        ip = cur_b;
-        ic = locate(sP, sL, S, ip);
+    // Position the dynamic issue cursor on its next tile; false when this
+    // worker has no more dynamic work.  Claims of kDynClaimTiles tiles are
+    // fired one claim ahead so that their latency hides behind streaming.
+    auto dyn_next_tile = [&]() -> bool {
+        for (int guard = 0; guard < 4 * nseg + 64; ++guard) {
+            if (dj >= 0 && d_t < d_te) {
+                if (!la_pending) {  // fire the next claim on this segment now
+                    if (lane == 0) la_val = epoch_add(p.dyn + (size_t)dj * kDynSegWords, kDynClaimTiles, epoch);
+                    la_pending = true;
+                }
+                return true;
+            }
+            if (dj >= 0) {
+                unsigned long long v = 0;
+                if (!la_pending && lane == 0) v = epoch_add(p.dyn + (size_t)dj * kDynSegWords, kDynClaimTiles, epoch);
+                if (la_pending && lane == 0) v = la_val;
+                la_pending = false;
+                v = __shfl_sync(kFull, v, 0);
+                if (v == ~0ull) {
+                    if (lane == 0) atomicOr(status, kFlagTimeout);
+                    return false;
+                }
+                const int t0 = (int)(unsigned)v;
+                if (t0 < d_ns) {
+                    d_t = t0;
+                    d_te = min(t0 + kDynClaimTiles, d_ns);
+                    continue;
+                }
+                dj = -1;  // segment exhausted: move on
+                if (d_k >= kDynPiecesPerWorker) return false;
+            }
+            // Find a segment with unclaimed tiles and free participant room:
+            // every lane peeks one candidate, so a round trip covers 32.
+            bool joined = false;
+            while (scan_left > 0 && !joined) {
+                const int span = nseg - part.Js;
+                // scan_left <= span, so a lane below scan_left wraps at most once.
+                const bool in_range = lane < scan_left;
+                int j = scan_j + lane;
+                if (j >= nseg) j -= span;
+                if (!in_range) j = part.Js;
+                const int s = j / Hkv;
+                const int ns = in_range ? tiles_of(sL[s]) : 0;
+                bool ok = in_range && ns > 0;
+                if (ok) {
+                    const unsigned long long pk = epoch_peek(p.dyn + (size_t)j * kDynSegWords, epoch);
+                    ok = (int)(unsigned)pk < ns && (int)(pk >> 32) < kDynPieceCap;
+                }
+                unsigned cand = __ballot_sync(kFull, ok);
+                while (cand != 0u && !joined) {
+                    const int src = __ffs(cand) - 1;
+                    cand &= cand - 1u;
+                    const int jj = __shfl_sync(kFull, j, src);
+                    const int ss = jj / Hkv, nss = tiles_of(sL[ss]);
+                    unsigned long long v = 0;
+                    if (lane == 0) v = epoch_join(p.dyn + (size_t)jj * kDynSegWords, kDynClaimTiles, kDynPieceCap, nss, epoch);
+                    v = __shfl_sync(kFull, v, 0);
+                    if (v == ~0ull) continue;
+                    const int idx = (int)(v >> 32), t0 = (int)(unsigned)v;
+                    dj = jj; d_s = ss; d_h = jj - ss * Hkv; d_ns = nss; d_reg = idx;
+                    d_t = t0; d_te = min(t0 + kDynClaimTiles, nss);
+                    d_kcur = d_k++;
+                    d_new = true;
+                    la_pending = false;
+                    joined = true;
+                    scan_j = jj;  // continue from here next time
+                }
+                if (!joined) {
+                    const int step = min(32, scan_left);
+                    scan_left -= step;
+                    scan_j += step;
+                    if (scan_j >= nseg) scan_j -= span;
+                } else {
+                    scan_left = span;  // a fresh full cycle after each join
+                }
+            }
+            if (!joined) return false;
+        }
+        return false;
     };
-    auto claim = [&]() {
-        if (lane == 0) claim_k = atomicAdd(p.ws_header + kHdrNextChunk, 1);
-        claim_pending = true;
+    auto position_next = [&]() -> bool {
+        if (mode == 0) {
+            if (ip < cur_e) {
+                nx_s = ic.s; nx_h = ic.h; nx_st = ic.st;
+                nx_new = ip == cur_b || ic.st == 0;
+                nx_piece = make_int4(ic.s, ic.h, cur_rid, ip == cur_b ? 1 : 0);
+                return true;
+            }
+            mode = part.D > 0 ? 1 : 2;
+        }
+        if (mode == 1) {
+            if (dyn_next_tile()) {
+                nx_s = d_s; nx_h = d_h; nx_st = d_t;
+                nx_new = d_new;
+                nx_piece = make_int4(d_s, d_h, -1 - d_kcur, d_reg);
+                return true;
+            }
+            mode = 2;
+        }
+        return false;
     };
-    // Move to the next range: the claimed dynamic chunk, if any.
-    auto next_range = [&]() -> bool {
-        if (part.K == 0) { issue_done = true; return false; }
-        if (!claim_pending) claim();
-        const int k = __shfl_sync(kFull, claim_k, 0);
-        claim_pending = false;
-        if (k >= part.K) { issue_done = true; return false; }
-        start_range(part.Ws + k);
-        return true;
-    };
-    auto issue_one = [&]() {
+    auto issue_next = [&]() {
         const int slot = issued % kStages;
-        const bool new_piece = ip == cur_b || ic.st == 0;
-        const int tok = ic.st * kTileTokens;
+        const int tok = nx_st * kTileTokens;
         const int j = tok / bs, tok0 = tok - j * bs, j0 = j & ~31;
-        if (win_s != ic.s || win_j0 != j0) {
-            if (pre_s == ic.s && pre_j0 == j0) {
+        if (win_s != nx_s || win_j0 != j0) {
+            if (pre_s == nx_s && pre_j0 == j0) {
                 win_v = pre_v; pre_s = -1;
             } else {
-                win_v = fetch_window(ic.s, j0);
+                win_v = fetch_window(nx_s, j0);
             }
-            win_s = ic.s; win_j0 = j0;
-            prefetch_next();
-        } else if (new_piece) {
-            prefetch_next();
+            win_s = nx_s; win_j0 = j0;
+            prefetch_next(nx_s, nx_h);
+        } else if (nx_new) {
+            prefetch_next(nx_s, nx_h);
         }
         const int pb = __shfl_sync(kFull, win_v, j - j0);
+        if (nx_new) ++pieces_issued;
         if (lane == 0) {
-            int row = pb * Hkv + ic.h;
+            int row = pb * Hkv + nx_h;
             if (pb < 0 || (long long)pb >= p.num_blocks) {
                 row = -1;  // fully out of bounds: TMA fills zeros
                 atomicOr(status, kFlagBadBlock);
             }
-            wmeta[slot] = make_int4(ip, cur_b, cur_e, cur_rid);
+            if (nx_new) wpieces[(pieces_issued - 1) & 3] = nx_piece;
+            wmeta[slot] = make_int4(nx_st, pieces_issued - 1, 0, 0);
             const uint32_t bar = smem_addr(&wbars[slot]);
             const uint32_t dst = smem_addr(wbase + slot * kStageBytes);
-            const uint32_t qbytes = new_piece ? (uint32_t)(g * kHeadDim * 2) : 0u;
+            const uint32_t qbytes = nx_new ? (uint32_t)(g * kHeadDim * 2) : 0u;
             fence_proxy_async_smem();
             mbar_arrive_expect_tx(bar, kStageBytes + qbytes);
             tma_load_3d(dst, &tmK, 0, tok0, row, bar);
             tma_load_3d(dst + kHalfBytes, &tmK, 64, tok0, row, bar);
             tma_load_3d(dst + kTileBytes, &tmV, 0, tok0, row, bar);
             tma_load_3d(dst + kTileBytes + kHalfBytes, &tmV, 64, tok0, row, bar);
-            if (new_piece) {
-                const uint16_t *qsrc = p.q + ((size_t)ic.s * p.num_q_heads + (size_t)ic.h * g) * kHeadDim;
-                bulk_load(smem_addr(qslots + (pieces_issued % kQSlots) * kQSlotBytes), qsrc, qbytes, bar);
+            if (nx_new) {
+                const uint16_t *qsrc = p.q + ((size_t)nx_s * p.num_q_heads + (size_t)nx_h * g) * kHeadDim;
+                bulk_load(smem_addr(qslots + ((pieces_issued - 1) % kQSlots) * kQSlotBytes), qsrc, qbytes, bar);
             }
         }
-        if (new_piece) ++pieces_issued;
         ++issued;
-        if (++ip < cur_e) advance(ic, sL, S, Hkv);
-        if (part.K > 0 && !claim_pending && cur_e - ip <= kClaimAhead) claim();
+        have_next = false;
+        if (mode == 0) {
+            if (++ip < cur_e) advance(ic, sL, S, Hkv);
+        } else {
+            ++d_t;
+            d_new = false;
+        }
     };
 
     // ---- consume side state ----
-    Cursor cc{0, 0, 0, 0};
-    int c_rid = 0, c_b = 0, c_e = 0;
-    int pieces_loaded = 0, piece_pos0 = 0;
-    bool piece_from_seg_start = false;
+    int cur_piece = -1, c_tiles = 0;
+    int4 cpi = make_int4(0, 0, 0, 0);
     uint32_t qf[16];
     float acc[8][4];
     float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
+    const int h0 = 2 * (lane & 3), h1 = h0 + 1;
+    const int trow = lane >> 2;  // token row of this lane in the S^T fragment
+    const int drow = lane >> 2;  // dim row of this lane in the O^T fragment
 
     auto refill = [&](int consumed) {
-        while (!issue_done && issued - consumed < kStages) {
-            if (ip >= cur_e) {
-                if (!next_range()) break;
-                continue;
+        while (issued - consumed < kStages) {
+            if (!have_next) {
+                have_next = position_next();
+                if (!have_next) break;
             }
-            const bool np_ = ip == cur_b || ic.st == 0;
-            if (np_ && pieces_issued >= pieces_loaded + kQSlots) break;
-            issue_one();
+            if (nx_new && pieces_issued >= cur_piece + 1 + kQSlots) break;  // query slot still in use
+            issue_next();
         }
     };
 
-    if (w < part.Ws) start_range(w);
-    const int h0 = 2 * (lane & 3), h1 = h0 + 1;
-    const int trow = lane >> 2;  // token row of this lane in the S^T fragment
+    // Finish the consume side's current piece: write its output, or leave its
+    // partial state and count its tiles, merging the segment if it was last.
+    auto finalize = [&]() {
+        float L0 = l0, L1 = l1;
+#pragma unroll
+        for (int o = 4; o < 32; o <<= 1) {
+            L0 += __shfl_xor_sync(kFull, L0, o);
+            L1 += __shfl_xor_sync(kFull, L1, o);
+        }
+        const int s = cpi.x, h = cpi.y;
+        const int ns = tiles_of(sL[s]);
+        if (c_tiles == ns) {
+            // One worker covered the whole segment: write the bf16 output rows.
+            uint16_t *o = p.out + ((size_t)s * p.num_q_heads + (size_t)h * g) * kHeadDim;
+            const float i0 = 1.f / L0, i1 = 1.f / L1;
+#pragma unroll
+            for (int mt = 0; mt < 8; ++mt) {
+                const int d = mt * 16 + drow;
+                if (h0 < g) {
+                    o[h0 * kHeadDim + d] = f2bf(acc[mt][0] * i0);
+                    o[h0 * kHeadDim + d + 8] = f2bf(acc[mt][2] * i0);
+                }
+                if (h1 < g) {
+                    o[h1 * kHeadDim + d] = f2bf(acc[mt][1] * i1);
+                    o[h1 * kHeadDim + d + 8] = f2bf(acc[mt][3] * i1);
+                }
+            }
+            return;
+        }
+        const bool is_static = cpi.z >= 0;
+        const size_t slotid = is_static ? 2 * (size_t)cpi.z + (cpi.w ? 0 : 1)
+                                        : 2 * (size_t)W + (size_t)w * kDynPiecesPerWorker + (size_t)(-1 - cpi.z);
+        float *A = p.ws_acc + slotid * kSlotFloats;
+#pragma unroll
+        for (int mt = 0; mt < 8; ++mt) {
+            const int d = mt * 16 + drow;
+            if (h0 < g) {
+                A[h0 * kHeadDim + d] = acc[mt][0];
+                A[h0 * kHeadDim + d + 8] = acc[mt][2];
+            }
+            if (h1 < g) {
+                A[h1 * kHeadDim + d] = acc[mt][1];
+                A[h1 * kHeadDim + d + 8] = acc[mt][3];
+            }
+        }
+        if (lane < 4) {
+            float *ML = p.ws_ml + slotid * kSlotMl;
+            ML[2 * h0] = m0; ML[2 * h0 + 1] = L0;
+            ML[2 * h1] = m1; ML[2 * h1 + 1] = L1;
+        }
+        const int seg = s * Hkv + h;
+        unsigned long long *dw = p.dyn + (size_t)seg * kDynSegWords;
+        if (!is_static && lane == 0)
+            dw[1 + cpi.w] = ((unsigned long long)epoch << 32) | (unsigned long long)slotid;
+        __threadfence();
+        __syncwarp();
+        int done = 0;
+        int *cnt = p.seg_done + seg;
+        if (lane == 0) done = atomicAdd(cnt, c_tiles) + c_tiles;
+        done = __shfl_sync(kFull, done, 0);
+        if (done != ns) return;
+        __threadfence();
+        const int a = sP[s] + h * ns;
+        if (is_static) {
+            const int r0 = part.range_of(a), r1 = part.range_of(a + ns - 1);
+            auto slot_static = [&](int i) -> size_t {
+                const int r = r0 + i;
+                return 2 * (size_t)r + (part.range_begin(r) < a ? 1 : 0);
+            };
+            merge_pieces(p, r1 - r0 + 1, slot_static, slot_static, s, h, lane);
+        } else {
+            // Registered participants that took tiles wrote their slot with
+            // this epoch; the others never wrote one.
+            const int nreg = min((int)(epoch_peek(dw, epoch) >> 32), kDynPieceCap);
+            unsigned long long e = lane < nreg ? __ldcg(dw + 1 + lane) : 0ull;
+            const bool valid = lane < nreg && (unsigned)(e >> 32) == epoch;
+            const unsigned mask = __ballot_sync(kFull, valid);
+            // Compact the valid slots into lanes 0 .. count-1 (count <= kDynPieceCap < 32).
+            int myslot = 0;
+            for (int k = 0; k < 32; ++k) {
+                const int src_slot = __shfl_sync(kFull, (int)(e & 0xffffffffull), k);
+                const bool src_valid = (mask >> k) & 1u;
+                const int dst = __popc(mask & ((1u << k) - 1));
+                if (src_valid && dst == lane) myslot = src_slot;
+            }
+            merge_pieces(
+                p, __popc(mask), [&](int) -> size_t { return (size_t)myslot; },
+                [&](int i) -> size_t { return (size_t)__shfl_sync(kFull, myslot, i); }, s, h, lane);
+        }
+        if (lane == 0) *cnt = 0;
+    };
+
     int consumed = 0;
     refill(0);
     while (consumed < issued) {
@@ -526,25 +770,17 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
             // Drain this worker's outstanding copies (bounded) before leaving.
             for (int k = consumed + 1; k < issued; ++k)
                 mbar_wait(smem_addr(&wbars[k % kStages]), (uint32_t)((k / kStages) & 1));
+            cur_piece = -1;
             break;
         }
         __syncwarp();
         const int4 meta = wmeta[slot];
-        const int pos = meta.x;
-        if (pos == meta.y) {
-            cc = locate(sP, sL, S, pos);
-            c_b = meta.y; c_e = meta.z; c_rid = meta.w;
-        } else {
-            advance(cc, sL, S, Hkv);
-        }
-        const uint8_t *stage = wbase + slot * kStageBytes;
-        const uint32_t sK = smem_addr(stage), sV = sK + kTileBytes;
-        const bool piece_start = pos == c_b || cc.st == 0;
-        const bool seg_last = cc.st == cc.ns - 1;
-        const bool piece_end = pos == c_e - 1 || seg_last;
-
-        if (piece_start) {
-            const uint32_t qs = smem_addr(qslots + (pieces_loaded % kQSlots) * kQSlotBytes);
+        const int st = meta.x, pord = meta.y;
+        if (pord != cur_piece) {
+            if (cur_piece >= 0) finalize();
+            cur_piece = pord;
+            cpi = wpieces[pord & 3];
+            const uint32_t qs = smem_addr(qslots + (pord % kQSlots) * kQSlotBytes);
 #pragma unroll
             for (int kp = 0; kp < 4; ++kp)
                 ldsm_x4(qs + (lane & 7) * (kHeadDim * 2) + (32 * kp + 8 * (lane >> 3)) * 2, qf[4 * kp], qf[4 * kp + 1],
@@ -553,14 +789,16 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
 #pragma unroll
                 for (int i = 0; i < 16; ++i) qf[i] = 0u;
             }
-            ++pieces_loaded;
-            piece_pos0 = pos;
-            piece_from_seg_start = cc.st == 0;
+            c_tiles = 0;
             m0 = m1 = -INFINITY;
             l0 = l1 = 0.f;
 #pragma unroll
             for (int mt = 0; mt < 8; ++mt) acc[mt][0] = acc[mt][1] = acc[mt][2] = acc[mt][3] = 0.f;
         }
+        const uint8_t *stage = wbase + slot * kStageBytes;
+        const uint32_t sK = smem_addr(stage), sV = sK + kTileBytes;
+        const int Ls = sL[cpi.x];
+        const int ns = tiles_of(Ls);
 
         // S^T (16 tokens x 8 heads) = K (16 x 128) . Q^T (128 x 8), two accumulation chains.
         float sa[4] = {0.f, 0.f, 0.f, 0.f}, sb[4] = {0.f, 0.f, 0.f, 0.f};
@@ -575,7 +813,7 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
                 else mma_bf16(sa, a0, a1, a2, a3, qf[2 * kk], qf[2 * kk + 1]);
             }
         }
-        const int n_valid = seg_last ? sL[cc.s] - (cc.ns - 1) * kTileTokens : kTileTokens;
+        const int n_valid = st == ns - 1 ? Ls - (ns - 1) * kTileTokens : kTileTokens;
         float x0 = (sa[0] + sb[0]) * p.scale_log2, x1 = (sa[1] + sb[1]) * p.scale_log2;
         float x2 = (sa[2] + sb[2]) * p.scale_log2, x3 = (sa[3] + sb[3]) * p.scale_log2;
         if (trow >= n_valid) x0 = x1 = -INFINITY;
@@ -627,80 +865,11 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
                 mma_bf16(acc[mt], a0, a1, a2, a3, pb0, pb1);
             }
         }
-
-        if (piece_end) {
-            float L0 = l0, L1 = l1;
-#pragma unroll
-            for (int o = 4; o < 32; o <<= 1) {
-                L0 += __shfl_xor_sync(kFull, L0, o);
-                L1 += __shfl_xor_sync(kFull, L1, o);
-            }
-            const int drow = lane >> 2;
-            if (piece_from_seg_start && seg_last) {
-                // One range covered the whole segment: write the bf16 output rows.
-                uint16_t *o = p.out + ((size_t)cc.s * p.num_q_heads + (size_t)cc.h * g) * kHeadDim;
-                const float i0 = 1.f / L0, i1 = 1.f / L1;
-#pragma unroll
-                for (int mt = 0; mt < 8; ++mt) {
-                    const int d = mt * 16 + drow;
-                    if (h0 < g) {
-                        o[h0 * kHeadDim + d] = f2bf(acc[mt][0] * i0);
-                        o[h0 * kHeadDim + d + 8] = f2bf(acc[mt][2] * i0);
-                    }
-                    if (h1 < g) {
-                        o[h1 * kHeadDim + d] = f2bf(acc[mt][1] * i1);
-                        o[h1 * kHeadDim + d + 8] = f2bf(acc[mt][3] * i1);
-                    }
-                }
-            } else {
-                // Cut by a range boundary: leave (m, l, acc) and count the tiles.
-                const size_t slotid = 2 * (size_t)c_rid + (piece_pos0 == c_b ? 0 : 1);
-                float *A = p.ws_acc + slotid * kSlotFloats;
-#pragma unroll
-                for (int mt = 0; mt < 8; ++mt) {
-                    const int d = mt * 16 + drow;
-                    if (h0 < g) {
-                        A[h0 * kHeadDim + d] = acc[mt][0];
-                        A[h0 * kHeadDim + d + 8] = acc[mt][2];
-                    }
-                    if (h1 < g) {
-                        A[h1 * kHeadDim + d] = acc[mt][1];
-                        A[h1 * kHeadDim + d + 8] = acc[mt][3];
-                    }
-                }
-                if (lane < 4) {
-                    float *ML = p.ws_ml + slotid * kSlotMl;
-                    ML[2 * h0] = m0; ML[2 * h0 + 1] = L0;
-                    ML[2 * h1] = m1; ML[2 * h1 + 1] = L1;
-                }
-                __threadfence();
-                __syncwarp();
-                int done = 0;
-                const int tiles = pos - piece_pos0 + 1;
-                int *cnt = p.seg_done + (size_t)cc.s * Hkv + cc.h;
-                if (lane == 0) done = atomicAdd(cnt, tiles) + tiles;
-                done = __shfl_sync(kFull, done, 0);
-                if (done == cc.ns) {
-                    __threadfence();
-                    const int a = sP[cc.s] + cc.h * cc.ns;
-                    merge_segment(p, part, a, a + cc.ns, cc.s, cc.h, lane);
-                    if (lane == 0) *cnt = 0;
-                }
-            }
-        }
+        ++c_tiles;
         ++consumed;
         refill(consumed);
     }
-    // The last warp to finish resets the chunk dispenser for the next call.
-    if (lane == 0) {
-        __threadfence();
-        const int n = atomicAdd(p.ws_header + kHdrWarpsDone, 1);
-        if (n == W - 1) {
-            p.ws_header[kHdrNextChunk] = 0;
-            p.ws_header[kHdrWarpsDone] = 0;
-            __threadfence();
-        }
-    }
+    if (cur_piece >= 0) finalize();
 }
 
 }  // namespace

@@ -148,6 +148,8 @@ extern "C" ps_status_t ps_decode_attention_noalloc(const void *q, const void *k_
     dp.out = static_cast<uint16_t *>(out);
     dp.ws_header = reinterpret_cast<int *>(ws);
     dp.seg_done = reinterpret_cast<int *>(ws + seg_off);
+    dp.dyn = nullptr;  // static split only: the dynamic state is never touched
+    dp.epoch = 1;
     dp.ws_acc = reinterpret_cast<float *>(ws + acc_off);
     dp.ws_ml = reinterpret_cast<float *>(ws + ml_off);
     dp.num_seqs = num_seqs;

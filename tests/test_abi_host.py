@@ -50,12 +50,13 @@ def test_plan_sizing_matches_layout():
         W = 152 * info["workers_per_cta"]
         assert info["max_workers"] == W
         assert info["dynamic_permille"] == 0
-        # header + per-segment counters (S x Hkv ints) + partial slots: two per static range
-        # and per dynamic chunk (at most 4 per worker), 8 heads x (128 acc + m, l) fp32 each
-        slots = 2 * W * 5
-        expect = 256 + 64 * 8 * 4 + slots * 8 * 128 * 4 + slots * 8 * 2 * 4
+        # header + per-segment counters (S x Hkv ints) + per-segment shared state (17 u64)
+        # + partial slots (2 per static range, 8 per worker for shared segments),
+        # 8 heads x (128 acc + m, l) fp32 each
+        slots = W * (2 + 8)
+        expect = 256 + 64 * 8 * 4 + 64 * 8 * 17 * 8 + slots * 8 * 128 * 4 + slots * 8 * 2 * 4
         assert ws == info["workspace_bytes"]
-        assert expect <= ws <= expect + 3 * 256
+        assert expect <= ws <= expect + 4 * 256
         assert info["smem_bytes"] <= 227 * 1024
     finally:
         psd.ps_decode_plan_destroy(plan)
