@@ -1,11 +1,13 @@
 #!/usr/bin/env python
 """Benchmark of paged GQA decode attention on GB300.
 
-One step = one decode-attention call (split-KV partial kernel + log-sum-exp
-combine) over one batch of a named synthetic workload whose inputs are
-already resident in HBM.  L2 is flushed (a 2x-L2 write) before every timed
-step, outside the timed interval, and each step is timed with CUDA events
-on the launching stream.
+One step = one decode-attention call (one kernel: the split-KV streaming
+pass with the log-sum-exp merge of cut pieces fused in) over one batch of a
+named synthetic workload whose inputs are already resident in HBM.  L2 is
+flushed before every timed step, outside the timed interval (a 2x-L2 buffer
+written and read back, so that no dirty lines are written back inside the
+next step), and each step is timed with CUDA events on the launching
+stream.
 
 Prints one JSON line.  Default workload: the Llama-3-8B-shaped decode layer
 (64 sequences, 32/8 heads, block 16, contexts U[1024, 4096]).  --config
@@ -56,8 +58,6 @@ def parse_args(argv=None):
                     help="L2 flush between steps: write a 2x-L2 buffer, then read it back so that "
                          "L2 holds clean lines (default), or only write it (leaves dirty lines whose "
                          "write-back lands inside the next timed step)")
-    ap.add_argument("--dynamic-permille", type=int, default=-1,
-                    help="share of the KV stream shared between warps at run time (-1: library default)")
     return ap.parse_args(argv)
 
 
@@ -251,7 +251,7 @@ def run_ours(args):
     lens = wl.seq_lens.cpu().numpy()
     alg = roofline.algorithmic_bytes(lens, wl.num_q_heads, wl.num_kv_heads, wl.head_dim, wl.block_size)
 
-    attn = ps_decode.DecodeAttention.for_workload(wl, dynamic_permille=args.dynamic_permille)
+    attn = ps_decode.DecodeAttention.for_workload(wl)
     out = torch.empty_like(wl.q)
     stream = torch.cuda.current_stream(dev)
     l2 = torch.cuda.get_device_properties(dev).L2_cache_size

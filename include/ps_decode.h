@@ -45,8 +45,8 @@
  *    used by two calls that can run concurrently; after a call that raised
  *    PS_DEVICE_TIMEOUT, hand the workspace to the plan again
  *    (ps_decode_plan_set_workspace) so that its counters are re-zeroed.
- *  - Results are deterministic: the split of the work depends only on the
- *    sequence lengths and the plan, never on scheduling.
+ *  - Results are bit-deterministic: the split of the work depends only on
+ *    the sequence lengths and the plan, never on scheduling.
  *  - A plan is not thread-safe: use it from one host thread at a time.
  */
 #ifndef PS_DECODE_H
@@ -83,9 +83,8 @@ typedef struct ps_decode_plan_info {
     int grid_ctas;             /* CTAs of the split-KV partial kernel */
     int workers_per_cta;       /* independent streaming warps per CTA */
     int stages_per_worker;     /* 16-token K/V tiles in flight per warp */
-    int max_workers;           /* cap on the static partition's worker count */
-    int min_stages_per_worker; /* floor on a static worker's share, in 16-token tiles */
-    int dynamic_permille;      /* share of the work handed out as dynamic chunks */
+    int max_workers;           /* cap on the number of equal ranges the work is split into */
+    int min_stages_per_worker; /* floor on a worker's share, in 16-token tiles */
     size_t workspace_bytes;
     size_t smem_bytes;         /* dynamic shared memory of the partial kernel */
 } ps_decode_plan_info_t;
@@ -111,25 +110,19 @@ ps_status_t ps_decode_plan_create(int num_seqs, int num_q_heads, int num_kv_head
                                   ps_decode_plan_t **plan, size_t *workspace_bytes);
 
 /*
- * As ps_decode_plan_create(), with explicit knobs (0 = default for the first
- * three, -1 = default for dynamic_permille):
+ * As ps_decode_plan_create(), with explicit knobs (0 = default for each):
  *   num_sms                SM count to size the grid for (0: query the device;
  *                          a positive value needs no GPU, e.g. for host tests)
- *   max_workers            upper bound on the number of equal static ranges
- *                          the batch's KV stream is split into
- *   min_stages_per_worker  smallest static range, in 16-token tiles
+ *   max_workers            upper bound on the number of equal contiguous
+ *                          ranges the batch's KV stream is split into
+ *                          (1 = one warp does everything, no split)
+ *   min_stages_per_worker  smallest range, in 16-token tiles
  *                          (1 = split as finely as the workers allow)
- *   dynamic_permille       share (0..1000) of the KV stream cut into small
- *                          fixed chunks that idle warps claim at run time;
- *                          0 = fully static split, -1 = default (0)
- * max_workers = 1 with dynamic_permille = 0 runs the whole batch in one
- * warp without any split.
  */
 ps_status_t ps_decode_plan_create_ex(int num_seqs, int num_q_heads, int num_kv_heads, int head_dim,
                                      int block_size, int max_blocks_per_seq, long long num_blocks,
                                      int num_sms, int max_workers, int min_stages_per_worker,
-                                     int dynamic_permille, ps_decode_plan_t **plan,
-                                     size_t *workspace_bytes);
+                                     ps_decode_plan_t **plan, size_t *workspace_bytes);
 
 /* Give the plan its caller-owned device workspace (>= workspace_bytes, 256-byte
  * aligned).  The first call after this zeroes the workspace's counters and

@@ -20,13 +20,12 @@ struct ps_decode_plan {
     uint32_t magic;
     int num_seqs, num_q_heads, num_kv_heads, head_dim, block_size, max_blocks_per_seq;
     long long num_blocks;
-    int num_sms, grid_ctas, max_workers, min_stages, dynamic_permille;
+    int num_sms, grid_ctas, max_workers, min_stages;
     size_t smem_bytes;
     WorkspaceLayout ws;
     void *workspace = nullptr;
     size_t workspace_size = 0;
     bool status_needs_clear = false;
-    unsigned epoch = 0;  // calls since the workspace was last zeroed; tags the dynamic state
     // TMA descriptors for the last (k_cache, v_cache) pair seen.
     const void *tm_k_ptr = nullptr, *tm_v_ptr = nullptr;
     alignas(64) CUtensorMap tmK;
@@ -119,11 +118,9 @@ ps_status_t run_planned(ps_decode_plan *p, const void *q, const void *k, const v
         p->tm_v_ptr = v;
     }
     uint8_t *ws = static_cast<uint8_t *>(p->workspace);
-    if (++p->epoch >= (1u << kEpochBits)) p->status_needs_clear = true;  // epoch wrapped: re-zero the workspace
     if (p->status_needs_clear) {
-        p->epoch = 1;
-        // Status word, chunk dispenser and per-segment counters start at zero;
-        // the kernel returns them to zero at the end of every call.
+        // The status word and the per-segment counters start at zero; the
+        // kernel returns the counters to zero at the end of every call.
         if (cudaMemsetAsync(ws, 0, p->ws.acc_off, st) != cudaSuccess) return PS_ERR_CUDA;
         p->status_needs_clear = false;
     }
@@ -135,8 +132,6 @@ ps_status_t run_planned(ps_decode_plan *p, const void *q, const void *k, const v
     dp.out = static_cast<uint16_t *>(out);
     dp.ws_header = reinterpret_cast<int *>(ws);
     dp.seg_done = reinterpret_cast<int *>(ws + p->ws.seg_done_off);
-    dp.dyn = reinterpret_cast<unsigned long long *>(ws + p->ws.dyn_off);
-    dp.epoch = p->epoch;
     dp.ws_acc = reinterpret_cast<float *>(ws + p->ws.acc_off);
     dp.ws_ml = reinterpret_cast<float *>(ws + p->ws.ml_off);
     dp.num_seqs = p->num_seqs;
@@ -149,7 +144,6 @@ ps_status_t run_planned(ps_decode_plan *p, const void *q, const void *k, const v
     dp.len_cap = p->max_blocks_per_seq * p->block_size;
     dp.max_workers = p->max_workers;
     dp.min_stages = p->min_stages;
-    dp.dynamic_permille = p->dynamic_permille;
     dp.scale_log2 = (float)((double)scale * 1.4426950408889634);
 
     if (p->ev_start && cudaEventRecord(p->ev_start, st) != cudaSuccess) return PS_ERR_CUDA;
@@ -165,14 +159,11 @@ extern "C" {
 
 ps_status_t ps_decode_plan_create_ex(int num_seqs, int num_q_heads, int num_kv_heads, int head_dim, int block_size,
                                      int max_blocks_per_seq, long long num_blocks, int num_sms, int max_workers,
-                                     int min_stages_per_worker, int dynamic_permille, ps_decode_plan_t **plan,
-                                     size_t *workspace_bytes) {
+                                     int min_stages_per_worker, ps_decode_plan_t **plan, size_t *workspace_bytes) {
     if (!plan || !workspace_bytes) return PS_ERR_INVALID_ARG;
     *plan = nullptr;
     *workspace_bytes = 0;
-    if (num_sms < 0 || max_workers < 0 || min_stages_per_worker < 0 || dynamic_permille < -1 ||
-        dynamic_permille > 1000)
-        return PS_ERR_INVALID_ARG;
+    if (num_sms < 0 || max_workers < 0 || min_stages_per_worker < 0) return PS_ERR_INVALID_ARG;
     ps_status_t e = check_shape(num_seqs, num_q_heads, num_kv_heads, head_dim, block_size, max_blocks_per_seq,
                                 num_blocks);
     if (e != PS_OK) return e;
@@ -197,7 +188,6 @@ ps_status_t ps_decode_plan_create_ex(int num_seqs, int num_q_heads, int num_kv_h
     const int total_workers = p->grid_ctas * kWorkersPerCta;
     p->max_workers = (max_workers > 0 && max_workers < total_workers) ? max_workers : total_workers;
     p->min_stages = min_stages_per_worker > 0 ? min_stages_per_worker : kDefaultMinStages;
-    p->dynamic_permille = dynamic_permille >= 0 ? dynamic_permille : kDefaultDynamicPermille;
     p->smem_bytes = partial_smem_bytes(num_seqs);
     p->ws = workspace_layout(num_seqs, num_kv_heads, total_workers);
     *plan = p;
@@ -209,7 +199,7 @@ ps_status_t ps_decode_plan_create(int num_seqs, int num_q_heads, int num_kv_head
                                   int max_blocks_per_seq, long long num_blocks, ps_decode_plan_t **plan,
                                   size_t *workspace_bytes) {
     return ps_decode_plan_create_ex(num_seqs, num_q_heads, num_kv_heads, head_dim, block_size, max_blocks_per_seq,
-                                    num_blocks, 0, 0, 0, -1, plan, workspace_bytes);
+                                    num_blocks, 0, 0, 0, plan, workspace_bytes);
 }
 
 ps_status_t ps_decode_plan_set_workspace(ps_decode_plan_t *plan, void *workspace, size_t bytes) {
@@ -260,7 +250,6 @@ ps_status_t ps_decode_plan_info(const ps_decode_plan_t *plan, ps_decode_plan_inf
     info->stages_per_worker = kStages;
     info->max_workers = plan->max_workers;
     info->min_stages_per_worker = plan->min_stages;
-    info->dynamic_permille = plan->dynamic_permille;
     info->workspace_bytes = plan->ws.total;
     info->smem_bytes = plan->smem_bytes;
     return PS_OK;

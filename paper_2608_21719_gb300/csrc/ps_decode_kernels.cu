@@ -6,17 +6,14 @@
 // Work layout.  The KV work of the whole batch is one "tape" of 16-token
 // tiles ordered by sequence, then KV head: segment (s, j) holds
 // ceil(L_s / 16) tiles.  Every CTA rebuilds the per-sequence prefix sums of
-// the tape in shared memory.  The first part of the tape is split into equal
-// contiguous static ranges, one per worker; the last part
-// (dynamic_permille / 1000 of it) is cut into fixed chunks that idle workers
-// claim from an atomic dispenser, so random per-SM and per-warp speed
-// differences are absorbed at the end instead of stretching the tail.  All
-// range boundaries are a fixed function of the lengths and the grid, so the
-// result does not depend on which warp ran which range.  The mix of short
-// answer-phase and long thinking-phase contexts (PowerSlider Sec. 2.2, Sec. 3
-// Obs. 3) therefore needs no host knowledge of the lengths.
+// the tape in shared memory from seq_lens, and worker w of Ws takes the
+// contiguous range [floor(w N / Ws), floor((w+1) N / Ws)) of the N tiles.
+// The split is balanced to one tile whatever the mix of short answer-phase
+// and long thinking-phase contexts (PowerSlider Sec. 2.2, Sec. 3 Obs. 3),
+// needs no host knowledge of the lengths and no atomics, and depends only on
+// the lengths and the grid, so results are bit-deterministic.
 //
-// Streaming.  A worker walks its ranges tile by tile.  Each tile's K and V
+// Streaming.  A worker walks its range tile by tile.  Each tile's K and V
 // page halves arrive by TMA (cp.async.bulk.tensor, 128-byte swizzle) in a
 // per-warp ring of shared-memory stages completed on mbarriers; each
 // (block, kv-head) page is read once for all g query heads of its group.
@@ -207,69 +204,15 @@ __device__ __forceinline__ void advance(Cursor &c, const int *sL, int S, int Hkv
     c.ns = c.s < S ? tiles_of(sL[c.s]) : 0;
 }
 
-// Split of the tape: static worker ranges over [0, Ns), then the dynamic
-// segments [Js, S*Hkv) (Ns is a segment start), shared at run time.
+// Split of the tape into Ws equal contiguous static ranges; range r covers
+// tiles [floor(r N / Ws), floor((r+1) N / Ws)).
 struct Partition {
-    int N, Ns, Ws, D, Js;
+    int N, Ws;
 
-    __device__ int range_of(int x) const { return (int)((((long long)x + 1) * Ws - 1) / Ns); }
-    __device__ int range_begin(int r) const { return (int)((long long)r * Ns / Ws); }
-    __device__ int range_end(int r) const { return (int)((long long)(r + 1) * Ns / Ws); }
+    __device__ int range_of(int x) const { return (int)((((long long)x + 1) * Ws - 1) / N); }
+    __device__ int range_begin(int r) const { return (int)((long long)r * N / Ws); }
+    __device__ int range_end(int r) const { return (int)((long long)(r + 1) * N / Ws); }
 };
-
-// Packed per-segment word: [epoch:20 | participants:12 | tile cursor:32].
-constexpr int kEpochShift = 64 - (int)kEpochBits;
-constexpr unsigned long long kJoinInc = 1ull << 32;
-
-// Add `inc` to a packed word and return its previous (participants, cursor)
-// part as seen in this call's epoch; a word still tagged with an older epoch
-// counts as zero.  Returns ~0 if the word could not be brought to the current
-// epoch within a bounded number of attempts.
-__device__ unsigned long long epoch_add(unsigned long long *w, unsigned long long inc, unsigned epoch) {
-    constexpr unsigned long long kValMask = (1ull << kEpochShift) - 1;
-    const unsigned long long tag = (unsigned long long)epoch << kEpochShift;
-    unsigned long long v = atomicAdd(w, inc);
-    if ((v & ~kValMask) == tag) return v & kValMask;
-    unsigned long long cur = v + inc;
-    for (int i = 0; i < 64; ++i) {
-        const unsigned long long prev = atomicCAS(w, cur, tag | inc);
-        if (prev == cur) return 0ull;
-        if ((prev & ~kValMask) == tag) {
-            v = atomicAdd(w, inc);
-            if ((v & ~kValMask) == tag) return v & kValMask;
-            cur = v + inc;
-        } else {
-            cur = prev;
-        }
-    }
-    return ~0ull;
-}
-
-// Join a shared segment and claim its next `claim` tiles in one step, but
-// only while it has fewer than `cap` participants and unclaimed tiles left
-// (a join past the cap must not take tiles it could not register).  Returns
-// the previous (participants, cursor) part, or ~0 if the segment is full,
-// exhausted, or kept changing for a bounded number of attempts.
-__device__ unsigned long long epoch_join(unsigned long long *w, unsigned claim, int cap, int ns, unsigned epoch) {
-    constexpr unsigned long long kValMask = (1ull << kEpochShift) - 1;
-    const unsigned long long tag = (unsigned long long)epoch << kEpochShift;
-    unsigned long long cur = __ldcg(w);
-    for (int i = 0; i < 64; ++i) {
-        const unsigned long long val = (cur & ~kValMask) == tag ? (cur & kValMask) : 0ull;
-        if ((int)(val >> 32) >= cap || (int)(unsigned)val >= ns) return ~0ull;
-        const unsigned long long prev = atomicCAS(w, cur, tag | (val + kJoinInc + claim));
-        if (prev == cur) return val;
-        cur = prev;
-    }
-    return ~0ull;
-}
-
-// (participants, cursor) part of a packed word in this call's epoch (0 if older).
-__device__ __forceinline__ unsigned long long epoch_peek(const unsigned long long *w, unsigned epoch) {
-    constexpr unsigned long long kValMask = (1ull << kEpochShift) - 1;
-    const unsigned long long v = __ldcg(w);
-    return (v >> kEpochShift) == epoch ? (v & kValMask) : 0ull;
-}
 
 // Merge `count` cut pieces of segment (s, h) into bf16 output rows by the
 // log-sum-exp rule.  Piece i's workspace slot comes from slot_lane(i), called
@@ -421,21 +364,10 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
     // 2. Partition of the tape (identical in every CTA).
     Partition part;
     const int W = gridDim.x * kWorkersPerCta;
-    const int nseg = S * Hkv;
     part.N = sP[S];
     {
-        const int dnom = p.dynamic_permille > 0 ? (int)((long long)part.N * p.dynamic_permille / 1000) : 0;
-        if (dnom > 0) {
-            const Cursor c = locate(sP, sL, S, part.N - dnom);  // round the split down to a segment start
-            part.Ns = sP[c.s] + c.h * c.ns;
-            part.Js = c.s * Hkv + c.h;
-        } else {
-            part.Ns = part.N;
-            part.Js = nseg;
-        }
-        part.D = part.N - part.Ns;
-        const int cap = (part.Ns + p.min_stages - 1) / p.min_stages;
-        part.Ws = part.Ns > 0 ? max(1, min(min(W, p.max_workers), cap)) : 0;
+        const int cap = (part.N + p.min_stages - 1) / p.min_stages;
+        part.Ws = part.N > 0 ? max(1, min(min(W, p.max_workers), cap)) : 0;
     }
     const int w = warp * gridDim.x + blockIdx.x;  // CTAs first: a small Ws still spreads over SMs
 
@@ -445,27 +377,17 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
     int4 *wmeta = metas + warp * kStages;
     int4 *wpieces = pieces + warp * 4;
     const int mbps = p.max_blocks_per_seq;
-    const unsigned epoch = p.epoch;
 
     // ---- issue side: TMA producer state (lane 0 issues, all lanes track) ----
-    // mode 0: static range, 1: dynamic segments, 2: nothing left to issue.
-    int mode = (w < part.Ws) ? 0 : (part.D > 0 ? 1 : 2);
-    int cur_rid = -1, cur_b = 0, cur_e = 0, ip = 0;
+    bool issuing = w < part.Ws;
+    int cur_rid = w, cur_b = 0, cur_e = 0, ip = 0;
     Cursor ic{0, 0, 0, 0};
-    if (mode == 0) {
-        cur_rid = w;
+    if (issuing) {
         cur_b = part.range_begin(w);
         cur_e = part.range_end(w);
         ip = cur_b;
         ic = locate(sP, sL, S, ip);
-        if (cur_b >= cur_e) mode = part.D > 0 ? 1 : 2;
     }
-    // dynamic-phase state
-    int dj = -1, d_s = 0, d_h = 0, d_ns = 0, d_t = 0, d_te = 0, d_reg = 0, d_k = 0, d_kcur = 0;
-    bool d_new = false, la_pending = false;
-    unsigned long long la_val = 0;  // lane 0: result of the claim fired ahead
-    int scan_j = part.Js + (int)((long long)w * (nseg - part.Js) / max(W, 1));
-    int scan_left = nseg - part.Js;
 
     int issued = 0, pieces_issued = 0;
     int win_s = -1, win_j0 = 0, win_v = -1;  // block-table window, one entry per lane
@@ -497,106 +419,12 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
         pre_s = ns_; pre_j0 = nj0;
         pre_v = fetch_window(ns_, nj0);
     };
-    // Position the dynamic issue cursor on its next tile; false when this
-    // worker has no more dynamic work.  Claims of kDynClaimTiles tiles are
-    // fired one claim ahead so that their latency hides behind streaming.
-    auto dyn_next_tile = [&]() -> bool {
-        for (int guard = 0; guard < 4 * nseg + 64; ++guard) {
-            if (dj >= 0 && d_t < d_te) {
-                if (!la_pending) {  // fire the next claim on this segment now
-                    if (lane == 0) la_val = epoch_add(p.dyn + (size_t)dj * kDynSegWords, kDynClaimTiles, epoch);
-                    la_pending = true;
-                }
-                return true;
-            }
-            if (dj >= 0) {
-                unsigned long long v = 0;
-                if (!la_pending && lane == 0) v = epoch_add(p.dyn + (size_t)dj * kDynSegWords, kDynClaimTiles, epoch);
-                if (la_pending && lane == 0) v = la_val;
-                la_pending = false;
-                v = __shfl_sync(kFull, v, 0);
-                if (v == ~0ull) {
-                    if (lane == 0) atomicOr(status, kFlagTimeout);
-                    return false;
-                }
-                const int t0 = (int)(unsigned)v;
-                if (t0 < d_ns) {
-                    d_t = t0;
-                    d_te = min(t0 + kDynClaimTiles, d_ns);
-                    continue;
-                }
-                dj = -1;  // segment exhausted: move on
-                if (d_k >= kDynPiecesPerWorker) return false;
-            }
-            // Find a segment with unclaimed tiles and free participant room:
-            // every lane peeks one candidate, so a round trip covers 32.
-            bool joined = false;
-            while (scan_left > 0 && !joined) {
-                const int span = nseg - part.Js;
-                // scan_left <= span, so a lane below scan_left wraps at most once.
-                const bool in_range = lane < scan_left;
-                int j = scan_j + lane;
-                if (j >= nseg) j -= span;
-                if (!in_range) j = part.Js;
-                const int s = j / Hkv;
-                const int ns = in_range ? tiles_of(sL[s]) : 0;
-                bool ok = in_range && ns > 0;
-                if (ok) {
-                    const unsigned long long pk = epoch_peek(p.dyn + (size_t)j * kDynSegWords, epoch);
-                    ok = (int)(unsigned)pk < ns && (int)(pk >> 32) < kDynPieceCap;
-                }
-                unsigned cand = __ballot_sync(kFull, ok);
-                while (cand != 0u && !joined) {
-                    const int src = __ffs(cand) - 1;
-                    cand &= cand - 1u;
-                    const int jj = __shfl_sync(kFull, j, src);
-                    const int ss = jj / Hkv, nss = tiles_of(sL[ss]);
-                    unsigned long long v = 0;
-                    if (lane == 0) v = epoch_join(p.dyn + (size_t)jj * kDynSegWords, kDynClaimTiles, kDynPieceCap, nss, epoch);
-                    v = __shfl_sync(kFull, v, 0);
-                    if (v == ~0ull) continue;
-                    const int idx = (int)(v >> 32), t0 = (int)(unsigned)v;
-                    dj = jj; d_s = ss; d_h = jj - ss * Hkv; d_ns = nss; d_reg = idx;
-                    d_t = t0; d_te = min(t0 + kDynClaimTiles, nss);
-                    d_kcur = d_k++;
-                    d_new = true;
-                    la_pending = false;
-                    joined = true;
-                    scan_j = jj;  // continue from here next time
-                }
-                if (!joined) {
-                    const int step = min(32, scan_left);
-                    scan_left -= step;
-                    scan_j += step;
-                    if (scan_j >= nseg) scan_j -= span;
-                } else {
-                    scan_left = span;  // a fresh full cycle after each join
-                }
-            }
-            if (!joined) return false;
-        }
-        return false;
-    };
     auto position_next = [&]() -> bool {
-        if (mode == 0) {
-            if (ip < cur_e) {
-                nx_s = ic.s; nx_h = ic.h; nx_st = ic.st;
-                nx_new = ip == cur_b || ic.st == 0;
-                nx_piece = make_int4(ic.s, ic.h, cur_rid, ip == cur_b ? 1 : 0);
-                return true;
-            }
-            mode = part.D > 0 ? 1 : 2;
-        }
-        if (mode == 1) {
-            if (dyn_next_tile()) {
-                nx_s = d_s; nx_h = d_h; nx_st = d_t;
-                nx_new = d_new;
-                nx_piece = make_int4(d_s, d_h, -1 - d_kcur, d_reg);
-                return true;
-            }
-            mode = 2;
-        }
-        return false;
+        if (!issuing || ip >= cur_e) return false;
+        nx_s = ic.s; nx_h = ic.h; nx_st = ic.st;
+        nx_new = ip == cur_b || ic.st == 0;
+        nx_piece = make_int4(ic.s, ic.h, cur_rid, ip == cur_b ? 1 : 0);
+        return true;
     };
     auto issue_next = [&]() {
         const int slot = issued % kStages;
@@ -639,12 +467,7 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
         }
         ++issued;
         have_next = false;
-        if (mode == 0) {
-            if (++ip < cur_e) advance(ic, sL, S, Hkv);
-        } else {
-            ++d_t;
-            d_new = false;
-        }
+        if (++ip < cur_e) advance(ic, sL, S, Hkv);
     };
 
     // ---- consume side state ----
@@ -697,9 +520,8 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
             }
             return;
         }
-        const bool is_static = cpi.z >= 0;
-        const size_t slotid = is_static ? 2 * (size_t)cpi.z + (cpi.w ? 0 : 1)
-                                        : 2 * (size_t)W + (size_t)w * kDynPiecesPerWorker + (size_t)(-1 - cpi.z);
+        // Cut by a range boundary: leave (m, l, acc) in the range's slot.
+        const size_t slotid = 2 * (size_t)cpi.z + (cpi.w ? 0 : 1);
         float *A = p.ws_acc + slotid * kSlotFloats;
 #pragma unroll
         for (int mt = 0; mt < 8; ++mt) {
@@ -718,45 +540,22 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
             ML[2 * h0] = m0; ML[2 * h0 + 1] = L0;
             ML[2 * h1] = m1; ML[2 * h1 + 1] = L1;
         }
-        const int seg = s * Hkv + h;
-        unsigned long long *dw = p.dyn + (size_t)seg * kDynSegWords;
-        if (!is_static && lane == 0)
-            dw[1 + cpi.w] = ((unsigned long long)epoch << 32) | (unsigned long long)slotid;
         __threadfence();
         __syncwarp();
         int done = 0;
-        int *cnt = p.seg_done + seg;
+        int *cnt = p.seg_done + (size_t)s * Hkv + h;
         if (lane == 0) done = atomicAdd(cnt, c_tiles) + c_tiles;
         done = __shfl_sync(kFull, done, 0);
         if (done != ns) return;
+        // This warp completed the segment: merge its pieces in tape order.
         __threadfence();
         const int a = sP[s] + h * ns;
-        if (is_static) {
-            const int r0 = part.range_of(a), r1 = part.range_of(a + ns - 1);
-            auto slot_static = [&](int i) -> size_t {
-                const int r = r0 + i;
-                return 2 * (size_t)r + (part.range_begin(r) < a ? 1 : 0);
-            };
-            merge_pieces(p, r1 - r0 + 1, slot_static, slot_static, s, h, lane);
-        } else {
-            // Registered participants that took tiles wrote their slot with
-            // this epoch; the others never wrote one.
-            const int nreg = min((int)(epoch_peek(dw, epoch) >> 32), kDynPieceCap);
-            unsigned long long e = lane < nreg ? __ldcg(dw + 1 + lane) : 0ull;
-            const bool valid = lane < nreg && (unsigned)(e >> 32) == epoch;
-            const unsigned mask = __ballot_sync(kFull, valid);
-            // Compact the valid slots into lanes 0 .. count-1 (count <= kDynPieceCap < 32).
-            int myslot = 0;
-            for (int k = 0; k < 32; ++k) {
-                const int src_slot = __shfl_sync(kFull, (int)(e & 0xffffffffull), k);
-                const bool src_valid = (mask >> k) & 1u;
-                const int dst = __popc(mask & ((1u << k) - 1));
-                if (src_valid && dst == lane) myslot = src_slot;
-            }
-            merge_pieces(
-                p, __popc(mask), [&](int) -> size_t { return (size_t)myslot; },
-                [&](int i) -> size_t { return (size_t)__shfl_sync(kFull, myslot, i); }, s, h, lane);
-        }
+        const int r0 = part.range_of(a), r1 = part.range_of(a + ns - 1);
+        auto slot_of = [&](int i) -> size_t {
+            const int r = r0 + i;
+            return 2 * (size_t)r + (part.range_begin(r) < a ? 1 : 0);
+        };
+        merge_pieces(p, r1 - r0 + 1, slot_of, slot_of, s, h, lane);
         if (lane == 0) *cnt = 0;
     };
 

@@ -119,7 +119,7 @@ extern "C" ps_status_t ps_decode_attention_noalloc(const void *q, const void *k_
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0)
         return PS_ERR_CUDA;
     // Scratch layout: header, per-segment counters, then two partial slots per
-    // static worker range (no dynamic chunks on this path).
+    // worker range, the layout the planned path uses.
     const int workers = sms * kWorkersPerCta;
     const size_t seg_off = kWsHeaderBytes;
     const size_t acc_off = align_up(seg_off + (size_t)num_seqs * num_kv_heads * 4, 256);
@@ -148,8 +148,6 @@ extern "C" ps_status_t ps_decode_attention_noalloc(const void *q, const void *k_
     dp.out = static_cast<uint16_t *>(out);
     dp.ws_header = reinterpret_cast<int *>(ws);
     dp.seg_done = reinterpret_cast<int *>(ws + seg_off);
-    dp.dyn = nullptr;  // static split only: the dynamic state is never touched
-    dp.epoch = 1;
     dp.ws_acc = reinterpret_cast<float *>(ws + acc_off);
     dp.ws_ml = reinterpret_cast<float *>(ws + ml_off);
     dp.num_seqs = num_seqs;
@@ -162,7 +160,6 @@ extern "C" ps_status_t ps_decode_attention_noalloc(const void *q, const void *k_
     dp.len_cap = (int)len_cap;
     dp.max_workers = workers;
     dp.min_stages = kDefaultMinStages;
-    dp.dynamic_permille = 0;
     dp.scale_log2 = (float)((double)scale * 1.4426950408889634);
     if (launch_decode(dp, tmK, tmV, sms, partial_smem_bytes(num_seqs), st) != cudaSuccess) return PS_ERR_CUDA;
     return PS_OK;

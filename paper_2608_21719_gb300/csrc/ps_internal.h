@@ -29,11 +29,7 @@ constexpr int kTileTokens = 16;     // tokens per streamed K/V tile (mma M = 16)
 constexpr int kWorkersPerCta = PS_WORKERS_PER_CTA;
 constexpr int kStages = PS_STAGES;
 constexpr int kQSlots = 2;               // query tiles staged per warp
-constexpr int kDefaultMinStages = 8;     // smallest static share of a worker, in tiles
-constexpr int kDefaultDynamicPermille = 0;    // tape share shared dynamically (opt-in)
-constexpr int kDynClaimTiles = 8;        // tiles per dynamic claim
-constexpr int kDynPieceCap = 16;         // workers that may share one dynamic segment
-constexpr int kDynPiecesPerWorker = 8;   // dynamic pieces one worker may leave
+constexpr int kDefaultMinStages = 8;     // smallest share of a worker, in tiles
 
 // Shared-memory geometry.  A 16-token x 128-dim bf16 tile is loaded as two
 // 64-column halves by TMA with 128-byte swizzle: [half][token][64].
@@ -49,30 +45,21 @@ constexpr size_t kWsHeaderBytes = 256;   // int32 words, see kHdr*
 constexpr int kHdrStatus = 0;            // PS_DEVICE_* flags (atomicOr)
 constexpr size_t kSlotFloats = (size_t)kMaxGroup * kHeadDim;  // acc of one partial piece
 constexpr size_t kSlotMl = (size_t)kMaxGroup * 2;              // (m, l) of one partial piece
-// Per-segment dynamic state, tagged with the call's epoch so that no call has
-// to reset it: one packed word [epoch:20 | participants:12 | tile cursor:32]
-// and a registry of kDynPieceCap words [epoch:32 | partial slot:32].
-constexpr size_t kDynSegWords = 1 + kDynPieceCap;
-constexpr unsigned kEpochBits = 20;      // epochs wrap (and the workspace is re-zeroed) at 2^20
-
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 struct WorkspaceLayout {
-    size_t seg_done_off, dyn_off, acc_off, ml_off, total;
+    size_t seg_done_off, acc_off, ml_off, total;
 };
 
-// Partial-piece slots: two per static worker range (its first and its last
-// piece) plus kDynPiecesPerWorker per worker for the dynamic phase.
-inline size_t max_slots(int total_workers) {
-    return (size_t)total_workers * (2 + kDynPiecesPerWorker);
-}
+// Partial-piece slots: two per worker range (its first and its last piece;
+// the pieces between them cover whole segments and need no slot).
+inline size_t max_slots(int total_workers) { return 2 * (size_t)total_workers; }
 
 inline WorkspaceLayout workspace_layout(int num_seqs, int num_kv_heads, int total_workers) {
     WorkspaceLayout w;
     const size_t segs = (size_t)num_seqs * num_kv_heads;
     w.seg_done_off = kWsHeaderBytes;
-    w.dyn_off = align_up(w.seg_done_off + segs * 4, 256);
-    w.acc_off = align_up(w.dyn_off + segs * kDynSegWords * 8, 256);
+    w.acc_off = align_up(w.seg_done_off + segs * 4, 256);
     const size_t slots = max_slots(total_workers);
     w.ml_off = align_up(w.acc_off + slots * kSlotFloats * 4, 256);
     w.total = align_up(w.ml_off + slots * kSlotMl * 4, 256);
@@ -91,16 +78,13 @@ struct DecodeParams {
     uint16_t *out;              // bf16 [S][Hq][128]
     int *ws_header;
     int *seg_done;              // [S][Hkv] tiles finished per segment (self-resetting)
-    unsigned long long *dyn;    // [S][Hkv][kDynSegWords] epoch-tagged dynamic state
     float *ws_acc;              // [slots][8][128]
     float *ws_ml;               // [slots][8][2]
     int num_seqs, num_q_heads, num_kv_heads, group, block_size, max_blocks_per_seq;
     long long num_blocks;
     int len_cap;                // max_blocks_per_seq * block_size
-    int max_workers;            // cap on static workers
-    int min_stages;             // floor on a static worker's share
-    int dynamic_permille;       // share of the tape shared dynamically
-    unsigned epoch;             // call counter (>= 1), tags the dynamic state
+    int max_workers;            // cap on workers
+    int min_stages;             // floor on a worker's share
     float scale_log2;           // scale * log2(e)
 };
 

@@ -49,8 +49,7 @@ class PlanInfo(ctypes.Structure):
         ("head_dim", ctypes.c_int), ("block_size", ctypes.c_int), ("max_blocks_per_seq", ctypes.c_int),
         ("num_blocks", ctypes.c_longlong), ("num_sms", ctypes.c_int), ("grid_ctas", ctypes.c_int),
         ("workers_per_cta", ctypes.c_int), ("stages_per_worker", ctypes.c_int), ("max_workers", ctypes.c_int),
-        ("min_stages_per_worker", ctypes.c_int), ("dynamic_permille", ctypes.c_int),
-        ("workspace_bytes", ctypes.c_size_t),
+        ("min_stages_per_worker", ctypes.c_int), ("workspace_bytes", ctypes.c_size_t),
         ("smem_bytes", ctypes.c_size_t),
     ]
 
@@ -63,7 +62,7 @@ _PLAN_DIMS = [_i, _i, _i, _i, _i, _i, ctypes.c_longlong]
 
 _SIGS = {
     "ps_decode_plan_create": (_i, _PLAN_DIMS + [ctypes.POINTER(_vp), ctypes.POINTER(_sz)]),
-    "ps_decode_plan_create_ex": (_i, _PLAN_DIMS + [_i, _i, _i, _i, ctypes.POINTER(_vp), ctypes.POINTER(_sz)]),
+    "ps_decode_plan_create_ex": (_i, _PLAN_DIMS + [_i, _i, _i, ctypes.POINTER(_vp), ctypes.POINTER(_sz)]),
     "ps_decode_plan_set_workspace": (_i, [_vp, _vp, _sz]),
     "ps_decode_plan_bind": (_i, [_vp, _vp]),
     "ps_decode_plan_destroy": (_i, [_vp]),
@@ -134,12 +133,11 @@ def ps_decode_plan_create(num_seqs, num_q_heads, num_kv_heads, head_dim, block_s
 
 
 def ps_decode_plan_create_ex(num_seqs, num_q_heads, num_kv_heads, head_dim, block_size, max_blocks_per_seq,
-                             num_blocks, num_sms=0, max_workers=0, min_stages_per_worker=0, dynamic_permille=-1):
+                             num_blocks, num_sms=0, max_workers=0, min_stages_per_worker=0):
     plan, ws = _vp(), _sz()
     _check(_lib.ps_decode_plan_create_ex(num_seqs, num_q_heads, num_kv_heads, head_dim, block_size,
                                          max_blocks_per_seq, num_blocks, num_sms, max_workers,
-                                         min_stages_per_worker, dynamic_permille, ctypes.byref(plan),
-                                         ctypes.byref(ws)),
+                                         min_stages_per_worker, ctypes.byref(plan), ctypes.byref(ws)),
            "ps_decode_plan_create_ex")
     return plan.value, ws.value
 
@@ -215,11 +213,11 @@ class DecodeAttention:
     """
 
     def __init__(self, num_seqs, num_q_heads, num_kv_heads, head_dim, block_size, max_blocks_per_seq,
-                 num_blocks, device=None, max_workers=0, min_stages_per_worker=0, dynamic_permille=-1):
+                 num_blocks, device=None, max_workers=0, min_stages_per_worker=0):
         import torch
         self.plan, self.ws_bytes = ps_decode_plan_create_ex(
             num_seqs, num_q_heads, num_kv_heads, head_dim, block_size, max_blocks_per_seq, num_blocks,
-            0, max_workers, min_stages_per_worker, dynamic_permille)
+            0, max_workers, min_stages_per_worker)
         self.workspace = torch.empty(self.ws_bytes, dtype=torch.uint8, device=device or "cuda")
         ps_decode_plan_set_workspace(self.plan, self.workspace, self.ws_bytes)
         self.shape = (num_seqs, num_q_heads, num_kv_heads, head_dim, block_size)

@@ -37,7 +37,7 @@ def test_status_strings_and_version():
 
 def _plan(**kw):
     args = dict(num_seqs=64, num_q_heads=32, num_kv_heads=8, head_dim=128, block_size=16, max_blocks_per_seq=256,
-                num_blocks=12000, num_sms=152, max_workers=0, min_stages_per_worker=0, dynamic_permille=-1)
+                num_blocks=12000, num_sms=152, max_workers=0, min_stages_per_worker=0)
     args.update(kw)
     return psd.ps_decode_plan_create_ex(**args)
 
@@ -49,12 +49,10 @@ def test_plan_sizing_matches_layout():
         assert info["grid_ctas"] == 152
         W = 152 * info["workers_per_cta"]
         assert info["max_workers"] == W
-        assert info["dynamic_permille"] == 0
-        # header + per-segment counters (S x Hkv ints) + per-segment shared state (17 u64)
-        # + partial slots (2 per static range, 8 per worker for shared segments),
+        # header + per-segment counters (S x Hkv ints) + two partial slots per worker range,
         # 8 heads x (128 acc + m, l) fp32 each
-        slots = W * (2 + 8)
-        expect = 256 + 64 * 8 * 4 + 64 * 8 * 17 * 8 + slots * 8 * 128 * 4 + slots * 8 * 2 * 4
+        slots = 2 * W
+        expect = 256 + 64 * 8 * 4 + slots * 8 * 128 * 4 + slots * 8 * 2 * 4
         assert ws == info["workspace_bytes"]
         assert expect <= ws <= expect + 4 * 256
         assert info["smem_bytes"] <= 227 * 1024
@@ -80,8 +78,6 @@ def test_max_seqs_plan_fits_shared_memory():
     (dict(num_seqs=4097), psd.PS_ERR_UNSUPPORTED),
     (dict(num_blocks=0), psd.PS_ERR_INVALID_ARG),
     (dict(num_sms=-1), psd.PS_ERR_INVALID_ARG),
-    (dict(dynamic_permille=1001), psd.PS_ERR_INVALID_ARG),
-    (dict(dynamic_permille=-2), psd.PS_ERR_INVALID_ARG),
 ])
 def test_plan_rejects_bad_shapes(kw, status):
     with pytest.raises(psd.PsError) as ei:
@@ -148,10 +144,9 @@ def test_stream_binding_lookup():
 
 
 def test_worker_overrides_are_recorded():
-    plan, _ = _plan(max_workers=1, min_stages_per_worker=3, dynamic_permille=0)
+    plan, _ = _plan(max_workers=1, min_stages_per_worker=3)
     try:
         info = psd.ps_decode_plan_info(plan)
         assert info["max_workers"] == 1 and info["min_stages_per_worker"] == 3
-        assert info["dynamic_permille"] == 0
     finally:
         psd.ps_decode_plan_destroy(plan)
