@@ -54,6 +54,8 @@ def parse_args(argv=None):
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="CPU time budget of the oracle baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--append", action="store_true",
+                    help="time the fused step: append the current token's K/V to the cache, then attend")
     ap.add_argument("--flush", choices=["write-read", "write"], default="write-read",
                     help="L2 flush between steps: write a 2x-L2 buffer, then read it back so that "
                          "L2 holds clean lines (default), or only write it (leaves dirty lines whose "
@@ -270,8 +272,18 @@ def run_ours(args):
 
     flush = _Flush
 
+    if args.append:
+        gen = torch.Generator(device=dev)
+        gen.manual_seed(cfg.seed + 77)
+        k_new = torch.randn((wl.num_seqs, wl.num_kv_heads, wl.head_dim), generator=gen, device=dev).to(torch.bfloat16)
+        v_new = torch.randn((wl.num_seqs, wl.num_kv_heads, wl.head_dim), generator=gen, device=dev).to(torch.bfloat16)
+
     def step():
-        attn(wl.q, wl.k_cache, wl.v_cache, wl.block_table, wl.seq_lens, out=out, scale=wl.scale, stream=stream)
+        if args.append:
+            attn.append(wl.q, k_new, v_new, wl.k_cache, wl.v_cache, wl.block_table, wl.seq_lens, out=out,
+                        scale=wl.scale, stream=stream)
+        else:
+            attn(wl.q, wl.k_cache, wl.v_cache, wl.block_table, wl.seq_lens, out=out, scale=wl.scale, stream=stream)
 
     for _ in range(max(args.warmup, 3)):
         flush.zero_()
@@ -362,6 +374,7 @@ def run_ours(args):
             "l2": "flushed before every step, outside the timed interval: %s of a %d MB buffer" % (
                 "write then read" if args.flush == "write-read" else "write", flush.nbytes >> 20),
             "parallelism": "replicas" if world == 1 else "dp%d (independent batches per GPU)" % world,
+            "step": "append current token K/V + attend" if args.append else "attend",
         },
         "frac_of_hbm_peak": round(alg["total"] / (ms_per_step * 1e-3) / 1e9 / hbm_peak, 4),
         "decode_tokens_per_s": round(wl.num_seqs * world * K / (total_ms * 1e-3), 1),

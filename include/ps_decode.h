@@ -168,6 +168,30 @@ ps_status_t ps_decode_attention_planned(const ps_decode_plan_t *plan, const void
                                         float scale, void *stream);
 
 /*
+ * One whole decode step of attention: append the current token's key and
+ * value to the paged cache and attend over every cached token including it
+ * (PowerSlider Sec. 2.2: each decode step adds one token per sequence and
+ * reads the whole KV cache).  One kernel launch.
+ *
+ *   k_new, v_new  bf16 [num_seqs][num_kv_heads][head_dim], 16-byte aligned:
+ *                 the current token's key and value
+ *   k_cache, v_cache  as in ps_decode_attention(), written in place: for
+ *                 every sequence with seq_lens[s] > 0, slot
+ *                 (seq_lens[s]-1) % block_size of block
+ *                 block_table[s][(seq_lens[s]-1) / block_size] receives the
+ *                 new rows (the caller has already counted the new token in
+ *                 seq_lens and reserved its block).  Nothing else in the
+ *                 cache is written.
+ * The result equals writing the rows first and then calling
+ * ps_decode_attention().  Errors as ps_decode_attention_planned(), plus
+ * PS_ERR_INVALID_ARG for a null or misaligned k_new / v_new.
+ */
+ps_status_t ps_decode_append_attention_planned(const ps_decode_plan_t *plan, const void *q, const void *k_new,
+                                               const void *v_new, void *k_cache, void *v_cache,
+                                               const int *block_table, const int *seq_lens, void *out,
+                                               float scale, void *stream);
+
+/*
  * Measurement hook: when events are set (cudaEvent_t as void*, NULL to
  * clear), every call records ev_start right before its kernel and ev_end
  * right after it, on the call's stream.

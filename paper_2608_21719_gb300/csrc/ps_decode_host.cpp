@@ -53,7 +53,7 @@ ps_status_t check_shape(int num_seqs, int num_q_heads, int num_kv_heads, int hea
     if (head_dim != kHeadDim) return PS_ERR_UNSUPPORTED;
     if (num_q_heads / num_kv_heads > kMaxGroup) return PS_ERR_UNSUPPORTED;
     if (block_size % kTileTokens != 0 || block_size > 256) return PS_ERR_UNSUPPORTED;
-    if (num_seqs > kMaxSeqs) return PS_ERR_UNSUPPORTED;
+    if (num_seqs > kMaxSeqs || partial_smem_bytes(num_seqs) > kMaxSmemPerCta) return PS_ERR_UNSUPPORTED;
     // Tile counts and TMA row coordinates are 32-bit.
     const long long len_cap = (long long)max_blocks_per_seq * block_size;
     const long long tiles = (long long)num_seqs * ((len_cap + kTileTokens - 1) / kTileTokens) * num_kv_heads;
@@ -98,8 +98,11 @@ ps_status_t encode_cache_map(CUtensorMap *tm, const void *base, const ps_decode_
 }
 
 ps_status_t run_planned(ps_decode_plan *p, const void *q, const void *k, const void *v, const int *bt,
-                        const int *sl, void *out, float scale, void *stream) {
+                        const int *sl, void *out, float scale, void *stream, const void *k_new = nullptr,
+                        const void *v_new = nullptr) {
     if (!q || !k || !v || !bt || !sl || !out) return PS_ERR_INVALID_ARG;
+    if ((k_new == nullptr) != (v_new == nullptr)) return PS_ERR_INVALID_ARG;
+    if (k_new && (!aligned(k_new, 16) || !aligned(v_new, 16))) return PS_ERR_INVALID_ARG;
     if (!aligned(q, 16) || !aligned(k, 16) || !aligned(v, 16) || !aligned(bt, 4) || !aligned(sl, 4) ||
         !aligned(out, 16))
         return PS_ERR_INVALID_ARG;
@@ -145,6 +148,10 @@ ps_status_t run_planned(ps_decode_plan *p, const void *q, const void *k, const v
     dp.max_workers = p->max_workers;
     dp.min_stages = p->min_stages;
     dp.scale_log2 = (float)((double)scale * 1.4426950408889634);
+    dp.k_new = static_cast<const uint16_t *>(k_new);
+    dp.v_new = static_cast<const uint16_t *>(v_new);
+    dp.k_cache_w = k_new ? static_cast<uint16_t *>(const_cast<void *>(k)) : nullptr;
+    dp.v_cache_w = k_new ? static_cast<uint16_t *>(const_cast<void *>(v)) : nullptr;
 
     if (p->ev_start && cudaEventRecord(p->ev_start, st) != cudaSuccess) return PS_ERR_CUDA;
     if (launch_decode(dp, p->tmK, p->tmV, p->grid_ctas, p->smem_bytes, st) != cudaSuccess) return PS_ERR_CUDA;
@@ -261,6 +268,16 @@ ps_status_t ps_decode_attention_planned(const ps_decode_plan_t *plan, const void
     if (!live(plan)) return PS_ERR_NO_PLAN;
     return run_planned(const_cast<ps_decode_plan *>(plan), q, k_cache, v_cache, block_table, seq_lens, out, scale,
                        stream);
+}
+
+ps_status_t ps_decode_append_attention_planned(const ps_decode_plan_t *plan, const void *q, const void *k_new,
+                                               const void *v_new, void *k_cache, void *v_cache,
+                                               const int *block_table, const int *seq_lens, void *out, float scale,
+                                               void *stream) {
+    if (!live(plan)) return PS_ERR_NO_PLAN;
+    if (!k_new || !v_new) return PS_ERR_INVALID_ARG;
+    return run_planned(const_cast<ps_decode_plan *>(plan), q, k_cache, v_cache, block_table, seq_lens, out, scale,
+                       stream, k_new, v_new);
 }
 
 ps_status_t ps_decode_attention(const void *q, const void *k_cache, const void *v_cache, const int *block_table,

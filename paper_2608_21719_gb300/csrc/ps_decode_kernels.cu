@@ -598,6 +598,29 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
         const uint32_t sK = smem_addr(stage), sV = sK + kTileBytes;
         const int Ls = sL[cpi.x];
         const int ns = tiles_of(Ls);
+        if (p.k_new != nullptr && st == ns - 1) {
+            // Fused append: the last token of the segment is the current one.
+            // Its K and V rows come from k_new / v_new (the cache slot still
+            // holds stale data in the tile TMA just delivered) and are also
+            // stored into the cache.  Lanes 0-15 move the K row, 16-31 the V
+            // row, one 16-byte chunk each.
+            const int tpos = Ls - 1;
+            const int r = tpos - (ns - 1) * kTileTokens;
+            const bool isv = lane >= 16;
+            const int ci = lane & 15, half = ci >> 3, c = ci & 7;
+            const size_t row = ((size_t)cpi.x * Hkv + cpi.y) * kHeadDim + (size_t)ci * 8;
+            const uint4 val = *reinterpret_cast<const uint4 *>((isv ? p.v_new : p.k_new) + row);
+            uint8_t *tile = const_cast<uint8_t *>(stage) + (isv ? kTileBytes : 0);
+            *reinterpret_cast<uint4 *>(tile + half * kHalfBytes + r * 128 + ((c ^ (r & 7)) << 4)) = val;
+            const int pb = __ldg(p.block_table + (size_t)cpi.x * mbps + tpos / bs);
+            if (pb >= 0 && (long long)pb < p.num_blocks) {
+                uint16_t *dst = (isv ? p.v_cache_w : p.k_cache_w) +
+                                (((size_t)pb * Hkv + cpi.y) * bs + tpos % bs) * kHeadDim + (size_t)ci * 8;
+                *reinterpret_cast<uint4 *>(dst) = val;
+            }
+            fence_proxy_async_smem();
+            __syncwarp();
+        }
 
         // S^T (16 tokens x 8 heads) = K (16 x 128) . Q^T (128 x 8), two accumulation chains.
         float sa[4] = {0.f, 0.f, 0.f, 0.f}, sb[4] = {0.f, 0.f, 0.f, 0.f};
@@ -675,16 +698,17 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
 
 cudaError_t launch_decode(const DecodeParams &p, const CUtensorMap &tmK, const CUtensorMap &tmV, int grid_ctas,
                           size_t smem_bytes, cudaStream_t stream) {
-    static bool attr_done[64] = {};
+    // Raise the kernel's dynamic shared-memory limit (per device) whenever a
+    // launch needs more than any earlier one did.
+    static size_t attr_bytes[64] = {};
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-    if (!attr_done[dev]) {
-        e = cudaFuncSetAttribute(ps_decode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)partial_smem_bytes(kMaxSeqs));
+    if (smem_bytes > attr_bytes[dev]) {
+        e = cudaFuncSetAttribute(ps_decode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_bytes);
         if (e != cudaSuccess) return e;
-        attr_done[dev] = true;
+        attr_bytes[dev] = smem_bytes;
     }
     ps_decode_kernel<<<grid_ctas, kWorkersPerCta * 32, smem_bytes, stream>>>(p, tmK, tmV);
     return cudaGetLastError();

@@ -107,7 +107,7 @@ extern "C" ps_status_t ps_decode_attention_noalloc(const void *q, const void *k_
         max_blocks_per_seq <= 0 || num_blocks <= 0 || num_q_heads % num_kv_heads != 0 || !std::isfinite(scale))
         return PS_ERR_INVALID_ARG;
     if (head_dim != kHeadDim || num_q_heads / num_kv_heads > kMaxGroup || block_size % kTileTokens != 0 ||
-        block_size > 256 || num_seqs > kMaxSeqs)
+        block_size > 256 || num_seqs > kMaxSeqs || partial_smem_bytes(num_seqs) > kMaxSmemPerCta)
         return PS_ERR_UNSUPPORTED;
     const long long len_cap = (long long)max_blocks_per_seq * block_size;
     if (len_cap > INT32_MAX || (long long)num_seqs * ((len_cap + kTileTokens - 1) / kTileTokens) * num_kv_heads > INT32_MAX ||
@@ -161,6 +161,8 @@ extern "C" ps_status_t ps_decode_attention_noalloc(const void *q, const void *k_
     dp.max_workers = workers;
     dp.min_stages = kDefaultMinStages;
     dp.scale_log2 = (float)((double)scale * 1.4426950408889634);
+    dp.k_new = dp.v_new = nullptr;
+    dp.k_cache_w = dp.v_cache_w = nullptr;
     if (launch_decode(dp, tmK, tmV, sms, partial_smem_bytes(num_seqs), st) != cudaSuccess) return PS_ERR_CUDA;
     return PS_OK;
 }

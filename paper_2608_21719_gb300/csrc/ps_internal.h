@@ -28,7 +28,10 @@ constexpr int kTileTokens = 16;     // tokens per streamed K/V tile (mma M = 16)
 #endif
 constexpr int kWorkersPerCta = PS_WORKERS_PER_CTA;
 constexpr int kStages = PS_STAGES;
-constexpr int kQSlots = 2;               // query tiles staged per warp
+#ifndef PS_QSLOTS
+#define PS_QSLOTS 2
+#endif
+constexpr int kQSlots = PS_QSLOTS;       // query tiles staged per warp
 constexpr int kDefaultMinStages = 8;     // smallest share of a worker, in tiles
 
 // Shared-memory geometry.  A 16-token x 128-dim bf16 tile is loaded as two
@@ -66,6 +69,8 @@ inline WorkspaceLayout workspace_layout(int num_seqs, int num_kv_heads, int tota
     return w;
 }
 
+constexpr size_t kMaxSmemPerCta = 227 * 1024;  // opt-in limit of one CTA on sm_100/sm_103
+
 inline size_t partial_smem_bytes(int num_seqs) {
     return 1024 /* alignment slack */ + (size_t)kWorkersPerCta * kWorkerBytes +
            (size_t)kWorkersPerCta * (kStages * (8 + 16) + 4 * 16) + (size_t)(2 * num_seqs + 1) * 4;
@@ -86,6 +91,10 @@ struct DecodeParams {
     int max_workers;            // cap on workers
     int min_stages;             // floor on a worker's share
     float scale_log2;           // scale * log2(e)
+    // Fused append (all null for plain decode attention): the current token's
+    // K and V, bf16 [S][Hkv][128], written into its cache slot and attended.
+    const uint16_t *k_new, *v_new;
+    uint16_t *k_cache_w, *v_cache_w;
 };
 
 // Launcher (ps_decode_kernels.cu).  Returns cudaSuccess or the launch error.

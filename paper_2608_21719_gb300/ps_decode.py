@@ -69,6 +69,7 @@ _SIGS = {
     "ps_decode_plan_info": (_i, [_vp, ctypes.POINTER(PlanInfo)]),
     "ps_decode_attention": (_i, [_vp, _vp, _vp, _vp, _vp, _vp, _i, _i, _i, _i, _i, _f, _vp]),
     "ps_decode_attention_planned": (_i, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _f, _vp]),
+    "ps_decode_append_attention_planned": (_i, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _f, _vp]),
     "ps_decode_plan_set_timing_events": (_i, [_vp, _vp, _vp]),
     "ps_decode_plan_read_device_status": (_i, [_vp, _vp, ctypes.POINTER(ctypes.c_uint)]),
     "ps_decode_attention_noalloc": (_i, [_vp, _vp, _vp, _vp, _vp, _vp, _i, _i, _i, _i, _i, _i, ctypes.c_longlong,
@@ -173,6 +174,14 @@ def ps_decode_attention_planned(plan, q, k_cache, v_cache, block_table, seq_lens
            "ps_decode_attention_planned")
 
 
+def ps_decode_append_attention_planned(plan, q, k_new, v_new, k_cache, v_cache, block_table, seq_lens, out,
+                                       scale, stream) -> None:
+    _check(_lib.ps_decode_append_attention_planned(plan, _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_cache),
+                                                   _ptr(v_cache), _ptr(block_table), _ptr(seq_lens), _ptr(out),
+                                                   float(scale), _stream(stream)),
+           "ps_decode_append_attention_planned")
+
+
 def ps_decode_attention_noalloc(q, k_cache, v_cache, block_table, seq_lens, out, num_seqs, num_q_heads,
                                 num_kv_heads, head_dim, block_size, max_blocks_per_seq, num_blocks, scale,
                                 stream) -> None:
@@ -239,6 +248,19 @@ class DecodeAttention:
         if stream is None:
             stream = torch.cuda.current_stream(q.device)
         ps_decode_attention_planned(self.plan, q, k_cache, v_cache, block_table, seq_lens, out, scale, stream)
+        return out
+
+    def append(self, q, k_new, v_new, k_cache, v_cache, block_table, seq_lens, out=None, scale=None, stream=None):
+        """Append the current token's K/V to the cache and attend (one launch)."""
+        import torch
+        if out is None:
+            out = torch.empty_like(q)
+        if scale is None:
+            scale = 1.0 / (q.shape[-1] ** 0.5)
+        if stream is None:
+            stream = torch.cuda.current_stream(q.device)
+        ps_decode_append_attention_planned(self.plan, q, k_new, v_new, k_cache, v_cache, block_table, seq_lens,
+                                           out, scale, stream)
         return out
 
     def device_status(self, stream=None) -> int:

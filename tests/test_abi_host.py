@@ -18,7 +18,8 @@ def test_every_declared_symbol_is_exported():
     names = psd.header_functions()
     expected = {"ps_decode_plan_create", "ps_decode_plan_create_ex", "ps_decode_plan_set_workspace",
                 "ps_decode_plan_bind", "ps_decode_plan_destroy", "ps_decode_plan_info", "ps_decode_attention",
-                "ps_decode_attention_planned", "ps_decode_plan_set_timing_events",
+                "ps_decode_attention_planned", "ps_decode_append_attention_planned",
+                "ps_decode_plan_set_timing_events",
                 "ps_decode_plan_read_device_status", "ps_decode_launch_count", "ps_status_string",
                 "ps_decode_abi_version"}
     assert expected <= set(names)
