@@ -45,6 +45,10 @@ def _bind(path: str):
     lib.ps_oracle_decode_attention.restype = i
     lib.ps_oracle_decode_attention_split.argtypes = common + [i, i, p]
     lib.ps_oracle_decode_attention_split.restype = i
+    lib.ps_oracle_kv_pack.argtypes = [p, p, p, i, p, i, i, i, i, ctypes.c_longlong, p, p]
+    lib.ps_oracle_kv_pack.restype = i
+    lib.ps_oracle_kv_unpack.argtypes = [p, p, p, i, p, i, i, i, i, ctypes.c_longlong, p, p]
+    lib.ps_oracle_kv_unpack.restype = i
     return lib
 
 
@@ -113,3 +117,47 @@ def decode_attention(q_bits, k_bits, v_bits, block_table, seq_lens, num_kv_heads
     if rc != 0:
         raise RuntimeError("oracle failed: %s (%d)" % (ERRORS.get(rc, "unknown"), rc))
     return out
+
+
+def packed_offsets(seq_lens, num_kv_heads: int, head_dim: int) -> np.ndarray:
+    """Element offsets of each sequence in a packed K/V hand-off buffer
+    (sequence i takes 2 * Hkv * L_i * d elements)."""
+    sizes = 2 * num_kv_heads * np.asarray(seq_lens, dtype=np.int64) * head_dim
+    return np.concatenate([[0], np.cumsum(sizes)[:-1]]).astype(np.int64)
+
+
+def kv_pack(k_bits, v_bits, block_table, seq_lens, offsets=None, lib=None) -> np.ndarray:
+    """Gather each sequence's K/V pages into the packed hand-off layout
+    [K: Hkv x L x d | V: Hkv x L x d] (bf16 bits, uint16)."""
+    lib = lib or load()
+    k = _as_u16(k_bits)
+    v = _as_u16(v_bits)
+    bt = np.ascontiguousarray(block_table, dtype=np.int32)
+    sl = np.ascontiguousarray(seq_lens, dtype=np.int32)
+    nb, hkv, bs, d = k.shape
+    off = packed_offsets(sl, hkv, d) if offsets is None else np.ascontiguousarray(offsets, dtype=np.int64)
+    total = int(off[-1] + 2 * hkv * int(sl[-1]) * d) if len(sl) else 0
+    dst = np.zeros(max(total, 1), dtype=np.uint16)
+    rc = lib.ps_oracle_kv_pack(k.ctypes.data, v.ctypes.data, bt.ctypes.data, bt.shape[1], sl.ctypes.data, len(sl),
+                               hkv, d, bs, nb, off.ctypes.data, dst.ctypes.data)
+    if rc != 0:
+        raise RuntimeError("oracle kv_pack failed: %s (%d)" % (ERRORS.get(rc, "unknown"), rc))
+    return dst[:total]
+
+
+def kv_unpack(packed, k_bits, v_bits, block_table, seq_lens, offsets=None, lib=None):
+    """Scatter a packed hand-off buffer into copies of the given caches
+    through block_table; returns (k, v) as uint16 arrays."""
+    lib = lib or load()
+    k = _as_u16(k_bits).copy()
+    v = _as_u16(v_bits).copy()
+    src = _as_u16(packed)
+    bt = np.ascontiguousarray(block_table, dtype=np.int32)
+    sl = np.ascontiguousarray(seq_lens, dtype=np.int32)
+    nb, hkv, bs, d = k.shape
+    off = packed_offsets(sl, hkv, d) if offsets is None else np.ascontiguousarray(offsets, dtype=np.int64)
+    rc = lib.ps_oracle_kv_unpack(src.ctypes.data, off.ctypes.data, bt.ctypes.data, bt.shape[1], sl.ctypes.data,
+                                 len(sl), hkv, d, bs, nb, k.ctypes.data, v.ctypes.data)
+    if rc != 0:
+        raise RuntimeError("oracle kv_unpack failed: %s (%d)" % (ERRORS.get(rc, "unknown"), rc))
+    return k, v

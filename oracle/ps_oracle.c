@@ -274,3 +274,79 @@ int ps_oracle_decode_attention_split(const uint16_t *q, const uint16_t *k_cache,
     jb.num_blocks = num_blocks; jb.scale = scale; jb.chunk_tokens = chunk_tokens; jb.out = out;
     return run(&jb, num_threads);
 }
+
+/*
+ * KV hand-off between stage pools (PowerSlider Sec. 5: a request's KV cache
+ * moves from the thinking pool to the answer pool; only the on-GPU gather and
+ * scatter are modelled here, not the transport).
+ *
+ * Packed layout of sequence i (element offset dst_offsets[i]):
+ *   K[j][t][:] for j < Hkv, t < L_i, then V[j][t][:] in the same order,
+ * i.e. 2 * Hkv * L_i * d contiguous bf16 elements.
+ *
+ * ps_oracle_kv_pack copies cache slot (block_table[i][t / bs], j, t % bs) to
+ * packed position (j, t); ps_oracle_kv_unpack copies it back through another
+ * block table.  Both return 0, -1 (invalid argument) or -2 (block id outside
+ * the pool); unpack leaves every slot it does not own untouched.
+ */
+static int kv_addr(const int32_t *bt, int mbps, long long nb, int hkv, int bs, int d, int i, int j, int t,
+                   size_t *off)
+{
+    int32_t b = bt[(size_t)i * mbps + t / bs];
+    if (b < 0 || (long long)b >= nb) return -2;
+    *off = (((size_t)b * hkv + (size_t)j) * bs + (size_t)(t % bs)) * d;
+    return 0;
+}
+
+int ps_oracle_kv_pack(const uint16_t *k_cache, const uint16_t *v_cache, const int32_t *block_table,
+                      int max_blocks_per_seq, const int32_t *seq_lens, int num_seqs, int num_kv_heads,
+                      int head_dim, int block_size, long long num_blocks, const long long *dst_offsets,
+                      uint16_t *dst)
+{
+    if (!k_cache || !v_cache || !block_table || !seq_lens || !dst_offsets || !dst || num_seqs < 0 ||
+        num_kv_heads <= 0 || head_dim <= 0 || block_size <= 0)
+        return -1;
+    for (int i = 0; i < num_seqs; ++i) {
+        const int L = seq_lens[i];
+        if (L < 0 || (long long)L > (long long)max_blocks_per_seq * block_size) return -1;
+        uint16_t *kd = dst + dst_offsets[i];
+        uint16_t *vd = kd + (size_t)num_kv_heads * L * head_dim;
+        for (int j = 0; j < num_kv_heads; ++j)
+            for (int t = 0; t < L; ++t) {
+                size_t off;
+                int e = kv_addr(block_table, max_blocks_per_seq, num_blocks, num_kv_heads, block_size, head_dim,
+                                i, j, t, &off);
+                if (e) return e;
+                size_t p = ((size_t)j * L + t) * head_dim;
+                memcpy(kd + p, k_cache + off, sizeof(uint16_t) * (size_t)head_dim);
+                memcpy(vd + p, v_cache + off, sizeof(uint16_t) * (size_t)head_dim);
+            }
+    }
+    return 0;
+}
+
+int ps_oracle_kv_unpack(const uint16_t *src, const long long *src_offsets, const int32_t *block_table,
+                        int max_blocks_per_seq, const int32_t *seq_lens, int num_seqs, int num_kv_heads,
+                        int head_dim, int block_size, long long num_blocks, uint16_t *k_cache, uint16_t *v_cache)
+{
+    if (!k_cache || !v_cache || !block_table || !seq_lens || !src_offsets || !src || num_seqs < 0 ||
+        num_kv_heads <= 0 || head_dim <= 0 || block_size <= 0)
+        return -1;
+    for (int i = 0; i < num_seqs; ++i) {
+        const int L = seq_lens[i];
+        if (L < 0 || (long long)L > (long long)max_blocks_per_seq * block_size) return -1;
+        const uint16_t *ks = src + src_offsets[i];
+        const uint16_t *vs = ks + (size_t)num_kv_heads * L * head_dim;
+        for (int j = 0; j < num_kv_heads; ++j)
+            for (int t = 0; t < L; ++t) {
+                size_t off;
+                int e = kv_addr(block_table, max_blocks_per_seq, num_blocks, num_kv_heads, block_size, head_dim,
+                                i, j, t, &off);
+                if (e) return e;
+                size_t p = ((size_t)j * L + t) * head_dim;
+                memcpy(k_cache + off, ks + p, sizeof(uint16_t) * (size_t)head_dim);
+                memcpy(v_cache + off, vs + p, sizeof(uint16_t) * (size_t)head_dim);
+            }
+    }
+    return 0;
+}

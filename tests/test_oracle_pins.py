@@ -261,3 +261,67 @@ def test_planted_mistake_is_caught(name, tmp_path):
     oracle.build(force=True, src=str(path), out=so)
     failed = _battery(oracle.load(so))
     assert failed, "planted mistake %s passed every pin" % name
+
+
+# --- KV hand-off pack / unpack -------------------------------------------
+
+def _handoff_case(seed, Hkv=2, d=16, bs=8, lens=(5, 0, 17, 8)):
+    gen = torch.Generator().manual_seed(seed)
+    kl = [torch.randn((L, Hkv, d), generator=gen).to(torch.bfloat16) for L in lens]
+    vl = [torch.randn((L, Hkv, d), generator=gen).to(torch.bfloat16) for L in lens]
+    L = np.asarray(lens, dtype=np.int32)
+    nb = inputs.blocks_needed(L, bs) + 3
+    bt = inputs.build_block_table(L, bs, max(1, int(L.max()) // bs + 2), nb, np.random.default_rng(seed))
+    k, v = inputs.scatter_logical(kl, vl, Hkv, bs, bt, nb)
+    return kl, vl, k, v, bt, L
+
+
+def test_pack_equals_logical_arrays():
+    kl, vl, k, v, bt, L = _handoff_case(61)
+    packed = oracle.kv_pack(inputs.bf16_bits(k), inputs.bf16_bits(v), bt, L)
+    off = oracle.packed_offsets(L, 2, 16)
+    for i, n in enumerate(L):
+        kp = packed[off[i]:off[i] + 2 * n * 16].reshape(2, n, 16)
+        vp = packed[off[i] + 2 * n * 16:off[i] + 4 * n * 16].reshape(2, n, 16)
+        assert np.array_equal(kp, inputs.bf16_bits(kl[i].permute(1, 0, 2)))
+        assert np.array_equal(vp, inputs.bf16_bits(vl[i].permute(1, 0, 2)))
+
+
+def test_unpack_into_another_pool_then_pack_round_trips():
+    kl, vl, k, v, bt, L = _handoff_case(62)
+    packed = oracle.kv_pack(inputs.bf16_bits(k), inputs.bf16_bits(v), bt, L)
+    # receiver: a different pool size and a different permutation
+    nb2 = inputs.blocks_needed(L, 8) + 9
+    bt2 = inputs.build_block_table(L, 8, bt.shape[1], nb2, np.random.default_rng(7))
+    k2 = np.full((nb2, 2, 8, 16), 0x7fc0, dtype=np.uint16)  # NaN everywhere
+    v2 = k2.copy()
+    k2u, v2u = oracle.kv_unpack(packed, k2, v2, bt2, L)
+    again = oracle.kv_pack(k2u, v2u, bt2, L)
+    assert np.array_equal(again, packed)
+    # slots that no sequence owns keep their old bits
+    owned = np.zeros(k2.shape[:1] + k2.shape[2:3], dtype=bool)
+    for i, n in enumerate(L):
+        for t in range(int(n)):
+            owned[bt2[i, t // 8], t % 8] = True
+    for b in range(nb2):
+        for t in range(8):
+            if not owned[b, t]:
+                assert np.all(k2u[b, :, t] == 0x7fc0) and np.all(v2u[b, :, t] == 0x7fc0)
+
+
+def test_pack_is_invariant_to_block_relabelling():
+    kl, vl, k, v, bt, L = _handoff_case(63)
+    a = oracle.kv_pack(inputs.bf16_bits(k), inputs.bf16_bits(v), bt, L)
+    nb = k.shape[0]
+    bt2 = inputs.build_block_table(L, 8, bt.shape[1], nb, np.random.default_rng(99))
+    k2, v2 = inputs.scatter_logical(kl, vl, 2, 8, bt2, nb)
+    b = oracle.kv_pack(inputs.bf16_bits(k2), inputs.bf16_bits(v2), bt2, L)
+    assert np.array_equal(a, b)
+
+
+def test_pack_rejects_block_outside_pool():
+    kl, vl, k, v, bt, L = _handoff_case(64)
+    bad = bt.copy()
+    bad[2, 1] = k.shape[0] + 3
+    with pytest.raises(RuntimeError, match="block id"):
+        oracle.kv_pack(inputs.bf16_bits(k), inputs.bf16_bits(v), bad, L)
