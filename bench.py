@@ -54,6 +54,8 @@ def parse_args(argv=None):
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="CPU time budget of the oracle baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--transfer", choices=["pack", "unpack"], default=None,
+                    help="time the KV hand-off gather (pack) or scatter (unpack) of the whole batch instead")
     ap.add_argument("--append", action="store_true",
                     help="time the fused step: append the current token's K/V to the cache, then attend")
     ap.add_argument("--flush", choices=["write-read", "write"], default="write-read",
@@ -418,6 +420,68 @@ def run_ours(args):
     return line
 
 
+# ------------------------------------------------------- KV hand-off ------
+
+def run_transfer(args):
+    """Pack (or unpack) every sequence of the workload between its paged pool
+    and contiguous per-sequence buffers; metric: bytes read + written / time."""
+    import numpy as np
+    import torch
+
+    from paper_2608_21719_gb300 import inputs, ps_decode
+
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    cfg = inputs.CONFIGS[args.config]
+    wl = inputs.make_workload(cfg, device=dev, poison=False)
+    lens = wl.seq_lens.cpu().numpy().astype(np.int64)
+    Hkv, d, bs = wl.num_kv_heads, wl.head_dim, wl.block_size
+    sizes = 2 * Hkv * lens * d
+    off = torch.from_numpy(np.concatenate([[0], np.cumsum(sizes)[:-1]]).astype(np.int64)).to(dev)
+    buf = torch.empty(int(sizes.sum()), dtype=torch.bfloat16, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    flush_buf = torch.empty(max(2 * l2, 64 << 20) // 4, dtype=torch.int32, device=dev)
+    sink = torch.empty((), dtype=torch.int32, device=dev)
+    args_common = (wl.block_table, wl.max_blocks_per_seq, wl.seq_lens, wl.num_seqs, Hkv, d, bs, wl.num_blocks)
+
+    def step():
+        if args.transfer == "pack":
+            ps_decode.ps_kv_pack(wl.k_cache, wl.v_cache, *args_common, off, buf, status, stream)
+        else:
+            ps_decode.ps_kv_unpack(buf, off, *args_common, wl.k_cache, wl.v_cache, status, stream)
+
+    for _ in range(max(args.warmup, 3)):
+        flush_buf.zero_(); torch.amax(flush_buf, dim=0, out=sink)
+        step()
+    torch.cuda.synchronize(dev)
+    K = args.steps
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    with ClockSampler(os.environ.get("CUDA_VISIBLE_DEVICES", "0").split(",")[0] or "0") as clk:
+        for a, b in ev:
+            flush_buf.zero_(); torch.amax(flush_buf, dim=0, out=sink)
+            a.record(stream)
+            step()
+            b.record(stream)
+        torch.cuda.synchronize(dev)
+    assert int(status.item()) == 0
+    ms = statistics.mean(a.elapsed_time(b) for a, b in ev)
+    moved = 2 * int(sizes.sum()) * 2  # every element read once and written once
+    peak, kind = measured_peaks()
+    gbs = moved / (ms * 1e-3) / 1e9
+    return {
+        "metric": "KV hand-off %s GB/s (read + write)" % args.transfer, "value": round(gbs, 2), "unit": "GB/s",
+        "n_gpus": 1, "steps": K, "warmup": args.warmup, "ms_per_step": round(ms, 5), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": cfg.name, "bytes_moved": moved, "l2": "write-then-read flush before every step"},
+        "roofline": {"kernel": "ps_kv_transfer_kernel", "bound": "hbm", "achieved": round(gbs, 1), "peak": peak,
+                     "peak_kind": kind + " (copy bandwidth)", "unit": "GB/s", "frac": round(gbs / peak, 4),
+                     "traffic": None},
+        "clocks": clk.summary(),
+    }
+
+
 # ------------------------------------------------------- reference arm ------
 
 def run_reference(args):
@@ -466,7 +530,12 @@ def run_reference(args):
 
 def main(argv=None):
     args = parse_args(argv)
-    line = run_reference(args) if args.impl == "reference" else run_ours(args)
+    if args.impl == "reference":
+        line = run_reference(args)
+    elif args.transfer:
+        line = run_transfer(args)
+    else:
+        line = run_ours(args)
     if line is not None:
         print(json.dumps(line), flush=True)
 

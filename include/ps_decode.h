@@ -192,6 +192,44 @@ ps_status_t ps_decode_append_attention_planned(const ps_decode_plan_t *plan, con
                                                float scale, void *stream);
 
 /*
+ * KV hand-off between stage pools (PowerSlider Sec. 5: a reasoning request's
+ * KV cache moves from the thinking pool to the answer pool).  These are the
+ * on-GPU gather and scatter on either side of the transfer; the transport is
+ * the caller's.  Neither needs a plan.
+ *
+ * Packed layout of sequence i, starting at element offset offsets[i] (int64,
+ * device array, a multiple of 8): K[j][t][0..head_dim) for kv head
+ * j < num_kv_heads and token t < seq_lens[i], then V in the same order, i.e.
+ * 2 * num_kv_heads * seq_lens[i] * head_dim bf16 elements.
+ *
+ * ps_kv_pack copies slot (block_table[i][t / block_size], j, t % block_size)
+ * of k_cache / v_cache to packed position (j, t).  ps_kv_unpack copies packed
+ * position (j, t) to that slot of the destination pool (block_table being the
+ * receiver's); slots of the pool that no packed token maps to are not written.
+ *
+ *   caches, dst/src  bf16, 16-byte aligned; cache layout as for decode
+ *   block_table      int32 [num_seqs][max_blocks_per_seq]
+ *   seq_lens         int32 [num_seqs] (values above max_blocks_per_seq *
+ *                    block_size are clamped; a sequence whose offset is not a
+ *                    multiple of 8 is skipped; both raise
+ *                    PS_DEVICE_LEN_CLAMPED)
+ *   num_blocks       blocks in the pool; out-of-pool ids skip their page and
+ *                    raise PS_DEVICE_BAD_BLOCK
+ *   device_status    optional device word that receives PS_DEVICE_* flags
+ * Supported: head_dim a multiple of 8, 1 <= num_seqs <= 4096.  Errors:
+ * PS_ERR_INVALID_ARG, PS_ERR_UNSUPPORTED, PS_ERR_CUDA.
+ */
+ps_status_t ps_kv_pack(const void *k_cache, const void *v_cache, const int *block_table,
+                       int max_blocks_per_seq, const int *seq_lens, int num_seqs, int num_kv_heads,
+                       int head_dim, int block_size, long long num_blocks, const long long *dst_offsets,
+                       void *dst, unsigned int *device_status, void *stream);
+
+ps_status_t ps_kv_unpack(const void *src, const long long *src_offsets, const int *block_table,
+                         int max_blocks_per_seq, const int *seq_lens, int num_seqs, int num_kv_heads,
+                         int head_dim, int block_size, long long num_blocks, void *k_cache, void *v_cache,
+                         unsigned int *device_status, void *stream);
+
+/*
  * Measurement hook: when events are set (cudaEvent_t as void*, NULL to
  * clear), every call records ev_start right before its kernel and ev_end
  * right after it, on the call's stream.

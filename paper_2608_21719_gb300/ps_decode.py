@@ -74,6 +74,8 @@ _SIGS = {
     "ps_decode_plan_read_device_status": (_i, [_vp, _vp, ctypes.POINTER(ctypes.c_uint)]),
     "ps_decode_attention_noalloc": (_i, [_vp, _vp, _vp, _vp, _vp, _vp, _i, _i, _i, _i, _i, _i, ctypes.c_longlong,
                                          _f, _vp]),
+    "ps_kv_pack": (_i, [_vp, _vp, _vp, _i, _vp, _i, _i, _i, _i, ctypes.c_longlong, _vp, _vp, _vp, _vp]),
+    "ps_kv_unpack": (_i, [_vp, _vp, _vp, _i, _vp, _i, _i, _i, _i, ctypes.c_longlong, _vp, _vp, _vp, _vp]),
     "ps_decode_launch_count": (ctypes.c_ulonglong, []),
     "ps_status_string": (ctypes.c_char_p, [_i]),
     "ps_decode_abi_version": (_i, []),
@@ -191,6 +193,20 @@ def ps_decode_attention_noalloc(q, k_cache, v_cache, block_table, seq_lens, out,
                                             _ptr(seq_lens), _ptr(out), num_seqs, num_q_heads, num_kv_heads,
                                             head_dim, block_size, max_blocks_per_seq, num_blocks, float(scale),
                                             _stream(stream)), "ps_decode_attention_noalloc")
+
+
+def ps_kv_pack(k_cache, v_cache, block_table, max_blocks_per_seq, seq_lens, num_seqs, num_kv_heads, head_dim,
+               block_size, num_blocks, dst_offsets, dst, device_status, stream) -> None:
+    _check(_lib.ps_kv_pack(_ptr(k_cache), _ptr(v_cache), _ptr(block_table), max_blocks_per_seq, _ptr(seq_lens),
+                           num_seqs, num_kv_heads, head_dim, block_size, num_blocks, _ptr(dst_offsets), _ptr(dst),
+                           _ptr(device_status), _stream(stream)), "ps_kv_pack")
+
+
+def ps_kv_unpack(src, src_offsets, block_table, max_blocks_per_seq, seq_lens, num_seqs, num_kv_heads, head_dim,
+                 block_size, num_blocks, k_cache, v_cache, device_status, stream) -> None:
+    _check(_lib.ps_kv_unpack(_ptr(src), _ptr(src_offsets), _ptr(block_table), max_blocks_per_seq, _ptr(seq_lens),
+                             num_seqs, num_kv_heads, head_dim, block_size, num_blocks, _ptr(k_cache), _ptr(v_cache),
+                             _ptr(device_status), _stream(stream)), "ps_kv_unpack")
 
 
 def ps_decode_plan_set_timing_events(plan, ev_start, ev_end) -> None:

@@ -21,7 +21,7 @@ def test_every_declared_symbol_is_exported():
                 "ps_decode_attention_planned", "ps_decode_append_attention_planned",
                 "ps_decode_plan_set_timing_events",
                 "ps_decode_plan_read_device_status", "ps_decode_launch_count", "ps_status_string",
-                "ps_decode_abi_version"}
+                "ps_decode_abi_version", "ps_decode_attention_noalloc", "ps_kv_pack", "ps_kv_unpack"}
     assert expected <= set(names)
     lib = ctypes.CDLL(psd.LIB_PATH)
     for n in names:
@@ -151,3 +151,19 @@ def test_worker_overrides_are_recorded():
         assert info["max_workers"] == 1 and info["min_stages_per_worker"] == 3
     finally:
         psd.ps_decode_plan_destroy(plan)
+
+
+def test_kv_transfer_validates_on_the_host():
+    off = 16
+    with pytest.raises(psd.PsError) as ei:  # null pointer
+        psd.ps_kv_pack(0, 16, 16, 4, 16, 2, 8, 128, 16, 100, off, 16, None, None)
+    assert ei.value.status == psd.PS_ERR_INVALID_ARG
+    with pytest.raises(psd.PsError) as ei:  # misaligned cache
+        psd.ps_kv_pack(8, 16, 16, 4, 16, 2, 8, 128, 16, 100, off, 16, None, None)
+    assert ei.value.status == psd.PS_ERR_INVALID_ARG
+    with pytest.raises(psd.PsError) as ei:  # head_dim not a multiple of 8
+        psd.ps_kv_unpack(16, off, 16, 4, 16, 2, 8, 100, 16, 100, 16, 16, None, None)
+    assert ei.value.status == psd.PS_ERR_UNSUPPORTED
+    with pytest.raises(psd.PsError) as ei:  # too many sequences
+        psd.ps_kv_unpack(16, off, 16, 4, 16, 5000, 8, 128, 16, 100, 16, 16, None, None)
+    assert ei.value.status == psd.PS_ERR_UNSUPPORTED
