@@ -238,11 +238,11 @@ class DecodeAttention:
     """
 
     def __init__(self, num_seqs, num_q_heads, num_kv_heads, head_dim, block_size, max_blocks_per_seq,
-                 num_blocks, device=None, max_workers=0, min_stages_per_worker=0):
+                 num_blocks, device=None, max_workers=0, min_stages_per_worker=0, num_sms=0):
         import torch
         self.plan, self.ws_bytes = ps_decode_plan_create_ex(
             num_seqs, num_q_heads, num_kv_heads, head_dim, block_size, max_blocks_per_seq, num_blocks,
-            0, max_workers, min_stages_per_worker)
+            num_sms, max_workers, min_stages_per_worker)
         self.workspace = torch.empty(self.ws_bytes, dtype=torch.uint8, device=device or "cuda")
         ps_decode_plan_set_workspace(self.plan, self.workspace, self.ws_bytes)
         self.shape = (num_seqs, num_q_heads, num_kv_heads, head_dim, block_size)
