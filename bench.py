@@ -56,6 +56,8 @@ def parse_args(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--transfer", choices=["pack", "unpack"], default=None,
                     help="time the KV hand-off gather (pack) or scatter (unpack) of the whole batch instead")
+    ap.add_argument("--min-stages", type=int, default=0,
+                    help="smallest share of one worker warp, in 16-token tiles (0: library default)")
     ap.add_argument("--sms", type=int, default=0,
                     help="size the persistent grid for this many SMs (0: all); a proxy for lower SM throughput")
     ap.add_argument("--append", action="store_true",
@@ -257,7 +259,7 @@ def run_ours(args):
     lens = wl.seq_lens.cpu().numpy()
     alg = roofline.algorithmic_bytes(lens, wl.num_q_heads, wl.num_kv_heads, wl.head_dim, wl.block_size)
 
-    attn = ps_decode.DecodeAttention.for_workload(wl, num_sms=args.sms)
+    attn = ps_decode.DecodeAttention.for_workload(wl, num_sms=args.sms, min_stages_per_worker=args.min_stages)
     out = torch.empty_like(wl.q)
     stream = torch.cuda.current_stream(dev)
     l2 = torch.cuda.get_device_properties(dev).L2_cache_size

@@ -32,7 +32,7 @@ constexpr int kStages = PS_STAGES;
 #define PS_QSLOTS 2
 #endif
 constexpr int kQSlots = PS_QSLOTS;       // query tiles staged per warp
-constexpr int kDefaultMinStages = 8;     // smallest share of a worker, in tiles
+constexpr int kDefaultMinStages = 2;     // smallest share of a worker, in tiles (tuned on the 4-sequence workload)
 
 // Shared-memory geometry.  A 16-token x 128-dim bf16 tile is loaded as two
 // 64-column halves by TMA with 128-byte swizzle: [half][token][64].
