@@ -8,7 +8,9 @@ library: no header, no helper, no constant.
 
 What the oracle computes is documented at the top of ``ps_oracle.c``: the
 decode-step attention of PowerSlider Sec. 2.2 over a block-table-paged KV
-cache, in the KV layout ``[num_blocks][num_kv_heads][block_size][head_dim]``.
+cache, in the KV layout ``[num_blocks][num_kv_heads][block_size][head_dim]``,
+plus the causal chunked-prefill form over the same cache and the KV hand-off
+pack/unpack gather and scatter.
 """
 from __future__ import annotations
 
@@ -45,6 +47,9 @@ def _bind(path: str):
     lib.ps_oracle_decode_attention.restype = i
     lib.ps_oracle_decode_attention_split.argtypes = common + [i, i, p]
     lib.ps_oracle_decode_attention_split.restype = i
+    lib.ps_oracle_prefill_attention.argtypes = [p, p, p, p, p, p, i, i, i, i, i, i, ctypes.c_longlong,
+                                                ctypes.c_double, i, p]
+    lib.ps_oracle_prefill_attention.restype = i
     lib.ps_oracle_kv_pack.argtypes = [p, p, p, i, p, i, i, i, i, ctypes.c_longlong, p, p]
     lib.ps_oracle_kv_pack.restype = i
     lib.ps_oracle_kv_unpack.argtypes = [p, p, p, i, p, i, i, i, i, ctypes.c_longlong, p, p]
@@ -161,3 +166,29 @@ def kv_unpack(packed, k_bits, v_bits, block_table, seq_lens, offsets=None, lib=N
     if rc != 0:
         raise RuntimeError("oracle kv_unpack failed: %s (%d)" % (ERRORS.get(rc, "unknown"), rc))
     return k, v
+
+
+def prefill_attention(q_bits, k_bits, v_bits, block_table, seq_lens, q_start, num_kv_heads: int, scale: float,
+                      num_threads: int | None = None, lib=None) -> np.ndarray:
+    """fp64 chunked-prefill attention.  q_bits [T, Hq, d] holds the new tokens
+    of every sequence (sequence s owns rows q_start[s] .. q_start[s+1]); they
+    are the last tokens of the seq_lens[s] cached ones and attend causally.
+    Returns out [T, Hq, d] float64."""
+    lib = lib or load()
+    q = _as_u16(q_bits)
+    k = _as_u16(k_bits)
+    v = _as_u16(v_bits)
+    bt = np.ascontiguousarray(block_table, dtype=np.int32)
+    sl = np.ascontiguousarray(seq_lens, dtype=np.int32)
+    qs = np.ascontiguousarray(q_start, dtype=np.int32)
+    T, Hq, d = q.shape
+    nb, hkv, bs, d2 = k.shape
+    if v.shape != k.shape or d2 != d or hkv != num_kv_heads or qs.shape != (len(sl) + 1,) or qs[-1] != T:
+        raise ValueError("inconsistent shapes")
+    out = np.empty((T, Hq, d), dtype=np.float64)
+    rc = lib.ps_oracle_prefill_attention(q.ctypes.data, k.ctypes.data, v.ctypes.data, bt.ctypes.data,
+                                         sl.ctypes.data, qs.ctypes.data, len(sl), Hq, hkv, d, bs, bt.shape[1], nb,
+                                         float(scale), int(num_threads or os.cpu_count() or 1), out.ctypes.data)
+    if rc != 0:
+        raise RuntimeError("oracle prefill failed: %s (%d)" % (ERRORS.get(rc, "unknown"), rc))
+    return out

@@ -43,6 +43,15 @@
  * GQA == MHA with repeated KV heads, and torch's fp64 scaled-dot-product
  * attention on tiny dense shapes.
  *
+ * ps_oracle_prefill_attention() is the chunked-prefill counterpart (query
+ * tokens that are the last Q_s cached tokens, causal); its pins are dense
+ * causal brute force, torch's fp64 causal scaled-dot-product attention on
+ * whole prompts, bit-exact equality with the decode oracle when Q_s = 1, and
+ * blindness to tokens after each query's position.
+ *
+ * ps_oracle_kv_pack()/ps_oracle_kv_unpack() are the KV hand-off gather and
+ * scatter (pure data movement, pinned bit-exact).
+ *
  * Error codes: 0 ok; -1 invalid argument; -2 a block id outside
  * [0, num_blocks) is referenced; -3 a sequence length exceeds
  * max_blocks_per_seq * block_size; -4 out of host memory.
@@ -349,4 +358,141 @@ int ps_oracle_kv_unpack(const uint16_t *src, const long long *src_offsets, const
             }
     }
     return 0;
+}
+
+/*
+ * Chunked-prefill attention over the paged cache (PowerSlider Sec. 2.2: the
+ * prefill phase processes many prompt tokens at once and is compute-bound,
+ * Sec. 3 Obs. 2).  Sequence s holds L_s = seq_lens[s] cached tokens, the last
+ * Q_s = q_start[s+1] - q_start[s] of which are the new (query) tokens; query i
+ * of sequence s sits at position p = L_s - Q_s + i and attends causally to the
+ * cached tokens t = 0 .. p:
+ *
+ *   out[q_start[s] + i][h] = sum_{t<=p} softmax_t(scale * q . K_s[t]) V_s[t]
+ *
+ * with KV head h / g and the same paged layout as decode.  q and out are
+ * [total query tokens][Hq][d].  With Q_s = 1 for every sequence this is
+ * exactly ps_oracle_decode_attention.  Error codes as for decode; -1 also for
+ * Q_s > L_s or a decreasing q_start.
+ */
+typedef struct {
+    const uint16_t *q, *k_cache, *v_cache;
+    const int32_t *block_table, *seq_lens, *q_start;
+    int num_seqs, num_q_heads, num_kv_heads, head_dim, block_size, max_blocks_per_seq;
+    long long num_blocks;
+    double scale;
+    double *out;
+    int total_q;
+    atomic_int next_row;
+    atomic_int status;
+} prefill_job_t;
+
+static int prefill_row(prefill_job_t *jb, int s, int i, int h, double *logits)
+{
+    const int d = jb->head_dim;
+    const int g = jb->num_q_heads / jb->num_kv_heads;
+    const int j = h / g;
+    const int L = jb->seq_lens[s];
+    const int Q = jb->q_start[s + 1] - jb->q_start[s];
+    const int p = L - Q + i;
+    const size_t row = (size_t)(jb->q_start[s] + i) * jb->num_q_heads + h;
+    const uint16_t *qv = jb->q + row * d;
+    double *o = jb->out + row * d;
+    job_t view;  /* reuse the decode address helper */
+    memset(&view, 0, sizeof view);
+    view.block_table = jb->block_table;
+    view.num_kv_heads = jb->num_kv_heads;
+    view.head_dim = d;
+    view.block_size = jb->block_size;
+    view.max_blocks_per_seq = jb->max_blocks_per_seq;
+    view.num_blocks = jb->num_blocks;
+    int err = 0;
+    for (int e = 0; e < d; ++e) o[e] = 0.0;
+    double m = -INFINITY;
+    for (int t = 0; t <= p; ++t) {
+        const uint16_t *kr = token_row(&view, jb->k_cache, s, j, t, &err);
+        if (err) return err;
+        double dot = 0.0;
+        for (int e = 0; e < d; ++e) dot += bf16_bits_to_double(qv[e]) * bf16_bits_to_double(kr[e]);
+        logits[t] = jb->scale * dot;
+        if (logits[t] > m) m = logits[t];
+    }
+    double z = 0.0;
+    for (int t = 0; t <= p; ++t) {
+        double w = exp(logits[t] - m);
+        z += w;
+        const uint16_t *vr = token_row(&view, jb->v_cache, s, j, t, &err);
+        if (err) return err;
+        for (int e = 0; e < d; ++e) o[e] += w * bf16_bits_to_double(vr[e]);
+    }
+    for (int e = 0; e < d; ++e) o[e] /= z;
+    return 0;
+}
+
+static void *prefill_worker(void *arg)
+{
+    prefill_job_t *jb = (prefill_job_t *)arg;
+    int maxL = 1;
+    for (int s = 0; s < jb->num_seqs; ++s)
+        if (jb->seq_lens[s] > maxL) maxL = jb->seq_lens[s];
+    double *logits = (double *)malloc(sizeof(double) * (size_t)maxL);
+    if (!logits) {
+        atomic_store(&jb->status, -4);
+        return NULL;
+    }
+    const int rows = jb->total_q * jb->num_q_heads;
+    for (;;) {
+        int r = atomic_fetch_add(&jb->next_row, 1);
+        if (r >= rows || atomic_load(&jb->status) != 0) break;
+        const int tok = r / jb->num_q_heads, h = r % jb->num_q_heads;
+        int s = 0;
+        while (jb->q_start[s + 1] <= tok) ++s;
+        int e = prefill_row(jb, s, tok - jb->q_start[s], h, logits);
+        if (e) {
+            int zero = 0;
+            atomic_compare_exchange_strong(&jb->status, &zero, e);
+            break;
+        }
+    }
+    free(logits);
+    return NULL;
+}
+
+int ps_oracle_prefill_attention(const uint16_t *q, const uint16_t *k_cache, const uint16_t *v_cache,
+                                const int32_t *block_table, const int32_t *seq_lens, const int32_t *q_start,
+                                int num_seqs, int num_q_heads, int num_kv_heads, int head_dim, int block_size,
+                                int max_blocks_per_seq, long long num_blocks, double scale, int num_threads,
+                                double *out)
+{
+    if (!q || !k_cache || !v_cache || !block_table || !seq_lens || !q_start || !out || num_seqs < 0 ||
+        num_q_heads <= 0 || num_kv_heads <= 0 || head_dim <= 0 || block_size <= 0 ||
+        num_q_heads % num_kv_heads != 0 || q_start[0] != 0)
+        return -1;
+    for (int s = 0; s < num_seqs; ++s) {
+        const int Q = q_start[s + 1] - q_start[s];
+        if (Q < 0 || Q > seq_lens[s]) return -1;
+        if ((long long)seq_lens[s] > (long long)max_blocks_per_seq * block_size) return -3;
+    }
+    prefill_job_t jb;
+    memset(&jb, 0, sizeof jb);
+    jb.q = q; jb.k_cache = k_cache; jb.v_cache = v_cache;
+    jb.block_table = block_table; jb.seq_lens = seq_lens; jb.q_start = q_start;
+    jb.num_seqs = num_seqs; jb.num_q_heads = num_q_heads; jb.num_kv_heads = num_kv_heads;
+    jb.head_dim = head_dim; jb.block_size = block_size; jb.max_blocks_per_seq = max_blocks_per_seq;
+    jb.num_blocks = num_blocks; jb.scale = scale; jb.out = out; jb.total_q = q_start[num_seqs];
+    atomic_init(&jb.next_row, 0);
+    atomic_init(&jb.status, 0);
+    if (num_threads < 1) num_threads = 1;
+    if (num_threads > 1024) num_threads = 1024;
+    pthread_t *tids = (pthread_t *)malloc(sizeof(pthread_t) * (size_t)num_threads);
+    if (!tids) return -4;
+    int started = 0;
+    for (int i = 0; i < num_threads; ++i) {
+        if (pthread_create(&tids[i], NULL, prefill_worker, &jb) != 0) break;
+        ++started;
+    }
+    if (started == 0) prefill_worker(&jb);
+    for (int i = 0; i < started; ++i) pthread_join(tids[i], NULL);
+    free(tids);
+    return atomic_load(&jb.status);
 }

@@ -325,3 +325,95 @@ def test_pack_rejects_block_outside_pool():
     bad[2, 1] = k.shape[0] + 3
     with pytest.raises(RuntimeError, match="block id"):
         oracle.kv_pack(inputs.bf16_bits(k), inputs.bf16_bits(v), bad, L)
+
+
+# --- chunked prefill -----------------------------------------------------
+
+def _prefill_case(seed, Hq=8, Hkv=2, d=32, bs=8, lens=(20, 9, 33), qlens=(7, 9, 1)):
+    gen = torch.Generator().manual_seed(seed)
+    kl = [torch.randn((L, Hkv, d), generator=gen).to(torch.bfloat16) for L in lens]
+    vl = [torch.randn((L, Hkv, d), generator=gen).to(torch.bfloat16) for L in lens]
+    T = int(sum(qlens))
+    q = torch.randn((T, Hq, d), generator=gen).to(torch.bfloat16)
+    L = np.asarray(lens, dtype=np.int32)
+    qs = np.concatenate([[0], np.cumsum(qlens)]).astype(np.int32)
+    nb = inputs.blocks_needed(L, bs) + 2
+    bt = inputs.build_block_table(L, bs, int(L.max()) // bs + 2, nb, np.random.default_rng(seed))
+    k, v = inputs.scatter_logical(kl, vl, Hkv, bs, bt, nb)
+    return q, kl, vl, k, v, bt, L, qs
+
+
+def _prefill_dense(q, kl, vl, L, qs, Hkv, scale):
+    T, Hq, d = q.shape
+    g = Hq // Hkv
+    out = np.zeros((T, Hq, d))
+    for s in range(len(L)):
+        K = kl[s].double().numpy()
+        V = vl[s].double().numpy()
+        Q = int(qs[s + 1] - qs[s])
+        for i in range(Q):
+            p = int(L[s]) - Q + i
+            for h in range(Hq):
+                x = scale * (K[:p + 1, h // g] @ q[qs[s] + i, h].double().numpy())
+                w = np.exp(x - x.max())
+                out[qs[s] + i, h] = (w[:, None] * V[:p + 1, h // g]).sum(0) / w.sum()
+    return out
+
+
+def test_prefill_matches_causal_brute_force():
+    q, kl, vl, k, v, bt, L, qs = _prefill_case(71)
+    got = oracle.prefill_attention(inputs.bf16_bits(q), inputs.bf16_bits(k), inputs.bf16_bits(v), bt, L, qs, 2, 0.2)
+    np.testing.assert_allclose(got, _prefill_dense(q, kl, vl, L, qs, 2, 0.2), rtol=1e-12, atol=1e-12)
+
+
+def test_prefill_with_one_query_per_sequence_is_decode_bit_exact():
+    q, kl, vl, k, v, bt, L, qs = _prefill_case(72, qlens=(1, 1, 1))
+    pre = oracle.prefill_attention(inputs.bf16_bits(q), inputs.bf16_bits(k), inputs.bf16_bits(v), bt, L, qs, 2, 0.3)
+    dec = oracle.decode_attention(inputs.bf16_bits(q), inputs.bf16_bits(k), inputs.bf16_bits(v), bt, L, 2, 0.3)
+    assert np.array_equal(pre, dec)
+
+
+def test_prefill_full_prompt_matches_torch_causal_sdpa():
+    lens = (24, 16)
+    q, kl, vl, k, v, bt, L, qs = _prefill_case(73, lens=lens, qlens=lens)
+    got = oracle.prefill_attention(inputs.bf16_bits(q), inputs.bf16_bits(k), inputs.bf16_bits(v), bt, L, qs, 2, 0.25)
+    for s in range(2):
+        Qs = q[qs[s]:qs[s + 1]].double().permute(1, 0, 2)[None]                 # [1, Hq, L, d]
+        Ks = kl[s].double().permute(1, 0, 2).repeat_interleave(4, 0)[None]
+        Vs = vl[s].double().permute(1, 0, 2).repeat_interleave(4, 0)[None]
+        ref = torch.nn.functional.scaled_dot_product_attention(Qs, Ks, Vs, is_causal=True, scale=0.25)
+        np.testing.assert_allclose(got[qs[s]:qs[s + 1]], ref[0].permute(1, 0, 2).numpy(), rtol=1e-12, atol=1e-12)
+
+
+def test_prefill_ignores_tokens_after_each_query():
+    q, kl, vl, k, v, bt, L, qs = _prefill_case(74, lens=(30,), qlens=(10,))
+    a = oracle.prefill_attention(inputs.bf16_bits(q), inputs.bf16_bits(k), inputs.bf16_bits(v), bt, L, qs, 2, 0.2)
+    # change K/V of the last 4 tokens: queries at positions < 26 must not move
+    kl2 = [kl[0].clone()]
+    vl2 = [vl[0].clone()]
+    kl2[0][26:] = 7.0
+    vl2[0][26:] = -5.0
+    k2, v2 = inputs.scatter_logical(kl2, vl2, 2, 8, bt, k.shape[0])
+    b = oracle.prefill_attention(inputs.bf16_bits(q), inputs.bf16_bits(k2), inputs.bf16_bits(v2), bt, L, qs, 2, 0.2)
+    assert np.array_equal(a[:6], b[:6])          # positions 20..25
+    assert not np.allclose(a[6:], b[6:])         # positions 26..29 see the change
+
+
+def test_planted_prefill_off_by_one_is_caught(tmp_path):
+    if shutil.which("gcc") is None:
+        pytest.skip("gcc not available")
+    src = open(os.path.join(os.path.dirname(oracle.__file__), "ps_oracle.c")).read()
+    mutated, n = re.subn(r"for \(int t = 0; t <= p; \+\+t\)", "for (int t = 0; t < p; ++t)", src)
+    assert n == 2
+    path = tmp_path / "mut.c"
+    path.write_text(mutated)
+    so = str(tmp_path / "libmut_prefill.so")
+    oracle.build(force=True, src=str(path), out=so)
+    q, kl, vl, k, v, bt, L, qs = _prefill_case(75)
+    try:
+        got = oracle.prefill_attention(inputs.bf16_bits(q), inputs.bf16_bits(k), inputs.bf16_bits(v), bt, L, qs, 2,
+                                       0.2, lib=oracle.load(so))
+        caught = not np.allclose(got, _prefill_dense(q, kl, vl, L, qs, 2, 0.2), rtol=1e-12, atol=1e-12)
+    except RuntimeError:
+        caught = True
+    assert caught
