@@ -230,6 +230,43 @@ ps_status_t ps_kv_unpack(const void *src, const long long *src_offsets, const in
                          unsigned int *device_status, void *stream);
 
 /*
+ * Chunked-prefill attention over the paged cache (PowerSlider Sec. 2.2: the
+ * prefill phase processes the new prompt tokens together and is compute-bound,
+ * Sec. 3 Obs. 2).  Sequence s owns query rows q_start[s] .. q_start[s+1]-1;
+ * they are the LAST Q_s = q_start[s+1] - q_start[s] of its seq_lens[s] cached
+ * tokens (their K/V are already in the cache), and query i of the sequence,
+ * at position p = seq_lens[s] - Q_s + i, attends to the cached tokens 0 .. p:
+ *
+ *   out[q_start[s] + i][h] = sum_{t <= p} softmax_t(scale * q . K_s[t]) V_s[t]
+ *
+ * with KV head h / g as for decode.  Q.K^T and P.V run on the tensor cores
+ * (tcgen05, fp32 accumulation in tensor memory); P is rounded to bf16.
+ *
+ *   q, out       bf16 [total_q_tokens][num_q_heads][head_dim], 16-byte aligned
+ *   k_cache, v_cache, block_table  as for ps_decode_attention()
+ *   seq_lens     int32 [num_seqs], tokens in the cache including the new ones
+ *   q_start      int32 [num_seqs + 1], q_start[0] = 0, non-decreasing,
+ *                q_start[num_seqs] <= total_q_tokens (all three on the device)
+ *   max_q_len    an upper bound on Q_s over the batch (sizes the grid; the
+ *                query tiles past a sequence's Q_s do nothing)
+ *   device_status  optional device word that receives PS_DEVICE_* flags
+ * A sequence with Q_s > seq_lens[s], a negative Q_s, a length above
+ * max_blocks_per_seq * block_size or rows outside [0, total_q_tokens) is
+ * skipped (its rows are not written) and raises PS_DEVICE_LEN_CLAMPED; an
+ * out-of-pool block id reads zeros and raises PS_DEVICE_BAD_BLOCK; a stalled
+ * pipeline gives up after ~2 s and raises PS_DEVICE_TIMEOUT.
+ * Supported: head_dim 128, g = num_q_heads / num_kv_heads <= 16, block_size a
+ * multiple of 16, num_seqs <= 65535.  Needs no workspace.  Errors:
+ * PS_ERR_INVALID_ARG (null or misaligned pointer, bad sizes, non-finite
+ * scale), PS_ERR_UNSUPPORTED, PS_ERR_CUDA.
+ */
+ps_status_t ps_prefill_attention(const void *q, const void *k_cache, const void *v_cache, const int *block_table,
+                                 const int *seq_lens, const int *q_start, void *out, int num_seqs,
+                                 int total_q_tokens, int max_q_len, int num_q_heads, int num_kv_heads,
+                                 int head_dim, int block_size, int max_blocks_per_seq, long long num_blocks,
+                                 float scale, unsigned int *device_status, void *stream);
+
+/*
  * Measurement hook: when events are set (cudaEvent_t as void*, NULL to
  * clear), every call records ev_start right before its kernel and ev_end
  * right after it, on the call's stream.

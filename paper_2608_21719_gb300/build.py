@@ -21,7 +21,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libps_decode.so")
-SOURCES = ["ps_decode_kernels.cu", "ps_decode_host.cpp", "ps_decode_noalloc.cu", "ps_kv_transfer.cu"]
+SOURCES = ["ps_decode_kernels.cu", "ps_decode_host.cpp", "ps_decode_noalloc.cu", "ps_kv_transfer.cu", "ps_prefill.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -262,3 +262,104 @@ def scatter_logical(k_logical: list, v_logical: list, num_kv_heads: int, block_s
 def bf16_bits(t: torch.Tensor) -> np.ndarray:
     """bf16 tensor -> numpy uint16 bit patterns (host copy)."""
     return t.detach().contiguous().cpu().view(torch.int16).numpy().view(np.uint16)
+
+
+# --- chunked prefill -------------------------------------------------------
+#
+# A prefill batch: sequence s already holds `prior` cached tokens (earlier
+# chunks of its prompt) and brings `new` prompt tokens whose K/V the serving
+# engine has written into the cache; the new tokens are the queries.  The
+# shapes follow the Llama-3-8B layer of the decode workloads; the chunk sizes
+# are those of chunked-prefill serving (hundreds to a few thousand tokens).
+
+@dataclass(frozen=True)
+class PrefillConfig:
+    key: str
+    name: str
+    num_seqs: int
+    num_q_heads: int
+    num_kv_heads: int
+    block_size: int
+    new_tokens: tuple    # (lo, hi) inclusive, uniform
+    prior_tokens: tuple  # (lo, hi) inclusive, uniform
+    seed: int
+    head_dim: int = HEAD_DIM
+
+
+PREFILL_CONFIGS = {
+    "p1": PrefillConfig(key="p1", name="tiny-prefill-gqa4", num_seqs=3, num_q_heads=8, num_kv_heads=2,
+                        block_size=16, new_tokens=(1, 300), prior_tokens=(0, 400), seed=10),
+    "p2": PrefillConfig(key="p2", name="llama3-8b-chunked-prefill", num_seqs=8, num_q_heads=32, num_kv_heads=8,
+                        block_size=16, new_tokens=(512, 2048), prior_tokens=(0, 4096), seed=11),
+}
+
+
+@dataclass
+class PrefillWorkload:
+    cfg: PrefillConfig | None
+    q: torch.Tensor            # [T, Hq, d] bf16, the new tokens of all sequences
+    k_cache: torch.Tensor      # [NB, Hkv, bs, d] bf16
+    v_cache: torch.Tensor
+    block_table: torch.Tensor  # [S, mbps] int32
+    seq_lens: torch.Tensor     # [S] int32, prior + new
+    q_start: torch.Tensor      # [S + 1] int32
+    q_lens: np.ndarray         # [S] int32 (host copy)
+    lengths: np.ndarray        # [S] int32 (host copy of seq_lens)
+    scale: float
+
+    @property
+    def max_q_len(self) -> int:
+        return int(self.q_lens.max(initial=0))
+
+    def to(self, device) -> "PrefillWorkload":
+        return PrefillWorkload(cfg=self.cfg, q=self.q.to(device), k_cache=self.k_cache.to(device),
+                               v_cache=self.v_cache.to(device), block_table=self.block_table.to(device),
+                               seq_lens=self.seq_lens.to(device), q_start=self.q_start.to(device),
+                               q_lens=self.q_lens, lengths=self.lengths, scale=self.scale)
+
+
+def make_prefill_workload(cfg: PrefillConfig | str, device="cpu", poison: bool = True,
+                          new=None, prior=None, num_q_heads: int | None = None,
+                          num_kv_heads: int | None = None, block_size: int | None = None,
+                          spare_blocks: int = 0, seed: int | None = None) -> PrefillWorkload:
+    """Build a prefill batch; `new` / `prior` override the sampled token
+    counts and the head / block sizes can be overridden for edge cases."""
+    if isinstance(cfg, str):
+        cfg = PREFILL_CONFIGS[cfg]
+    seed = cfg.seed if seed is None else seed
+    Hq = num_q_heads or cfg.num_q_heads
+    Hkv = num_kv_heads or cfg.num_kv_heads
+    bs = block_size or cfg.block_size
+    rng = np.random.default_rng(seed)
+    if new is None:
+        new = rng.integers(cfg.new_tokens[0], cfg.new_tokens[1], size=cfg.num_seqs, endpoint=True)
+    if prior is None:
+        prior = rng.integers(cfg.prior_tokens[0], cfg.prior_tokens[1], size=len(new), endpoint=True)
+    q_lens = np.asarray(new, dtype=np.int32)
+    lengths = (np.asarray(prior, dtype=np.int64) + q_lens).astype(np.int32)
+    S = len(lengths)
+    mbps = max(1, (int(lengths.max(initial=0)) + bs - 1) // bs)
+    num_blocks = max(1, blocks_needed(lengths, bs) + spare_blocks)
+    bt = build_block_table(lengths, bs, mbps, num_blocks, np.random.default_rng(seed + 1000))
+    device = torch.device(device)
+    gen = torch.Generator(device=device)
+    gen.manual_seed(int(seed))
+    T = int(q_lens.sum())
+    q = torch.randn((T, Hq, cfg.head_dim), generator=gen, device=device, dtype=torch.float32).to(torch.bfloat16)
+    shape = (num_blocks, Hkv, bs, cfg.head_dim)
+    k = torch.empty(shape, device=device, dtype=torch.bfloat16)
+    v = torch.empty(shape, device=device, dtype=torch.bfloat16)
+    slab = max(1, (1 << 26) // (Hkv * bs * cfg.head_dim))
+    for t in (k, v):
+        for b0 in range(0, num_blocks, slab):
+            b1 = min(num_blocks, b0 + slab)
+            t[b0:b1] = torch.randn((b1 - b0,) + shape[1:], generator=gen, device=device,
+                                   dtype=torch.float32).to(torch.bfloat16)
+    if poison:
+        poison_unused(k, v, bt, lengths)
+    q_start = np.concatenate([[0], np.cumsum(q_lens)]).astype(np.int32)
+    return PrefillWorkload(cfg=cfg, q=q, k_cache=k, v_cache=v,
+                           block_table=torch.from_numpy(bt).to(device),
+                           seq_lens=torch.from_numpy(np.ascontiguousarray(lengths)).to(device),
+                           q_start=torch.from_numpy(q_start).to(device), q_lens=q_lens, lengths=lengths,
+                           scale=1.0 / math.sqrt(cfg.head_dim))

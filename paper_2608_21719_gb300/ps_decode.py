@@ -76,6 +76,8 @@ _SIGS = {
                                          _f, _vp]),
     "ps_kv_pack": (_i, [_vp, _vp, _vp, _i, _vp, _i, _i, _i, _i, ctypes.c_longlong, _vp, _vp, _vp, _vp]),
     "ps_kv_unpack": (_i, [_vp, _vp, _vp, _i, _vp, _i, _i, _i, _i, ctypes.c_longlong, _vp, _vp, _vp, _vp]),
+    "ps_prefill_attention": (_i, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _i, _i, _i, _i, _i, _i, _i, _i,
+                                  ctypes.c_longlong, _f, _vp, _vp]),
     "ps_decode_launch_count": (ctypes.c_ulonglong, []),
     "ps_status_string": (ctypes.c_char_p, [_i]),
     "ps_decode_abi_version": (_i, []),
@@ -207,6 +209,33 @@ def ps_kv_unpack(src, src_offsets, block_table, max_blocks_per_seq, seq_lens, nu
     _check(_lib.ps_kv_unpack(_ptr(src), _ptr(src_offsets), _ptr(block_table), max_blocks_per_seq, _ptr(seq_lens),
                              num_seqs, num_kv_heads, head_dim, block_size, num_blocks, _ptr(k_cache), _ptr(v_cache),
                              _ptr(device_status), _stream(stream)), "ps_kv_unpack")
+
+
+def ps_prefill_attention(q, k_cache, v_cache, block_table, seq_lens, q_start, out, num_seqs, total_q_tokens,
+                         max_q_len, num_q_heads, num_kv_heads, head_dim, block_size, max_blocks_per_seq, num_blocks,
+                         scale, device_status, stream) -> None:
+    _check(_lib.ps_prefill_attention(_ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(block_table), _ptr(seq_lens),
+                                     _ptr(q_start), _ptr(out), num_seqs, total_q_tokens, max_q_len, num_q_heads,
+                                     num_kv_heads, head_dim, block_size, max_blocks_per_seq, num_blocks, scale,
+                                     _ptr(device_status), _stream(stream)), "ps_prefill_attention")
+
+
+def prefill_attention(q, k_cache, v_cache, block_table, seq_lens, q_start, max_q_len, out=None, scale=None,
+                      device_status=None, stream=None):
+    """Tensor-level wrapper: q [T, Hq, 128] bf16 on the GPU, caches
+    [num_blocks, Hkv, bs, 128], block_table [S, mbps] int32, seq_lens [S]
+    int32, q_start [S + 1] int32.  Returns out [T, Hq, 128] bf16."""
+    import torch
+    T, Hq, d = q.shape
+    nb, hkv, bs, _ = k_cache.shape
+    if out is None:
+        out = torch.empty_like(q)
+    if scale is None:
+        scale = d ** -0.5
+    ps_prefill_attention(q, k_cache, v_cache, block_table, seq_lens, q_start, out, seq_lens.shape[0], T,
+                         int(max_q_len), Hq, hkv, d, bs, block_table.shape[1], nb, float(scale), device_status,
+                         stream)
+    return out
 
 
 def ps_decode_plan_set_timing_events(plan, ev_start, ev_end) -> None:

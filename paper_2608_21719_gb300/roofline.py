@@ -39,3 +39,24 @@ def decode_flops(seq_lens, num_q_heads: int, head_dim: int) -> int:
     """Q.K^T and P.V multiply-adds, 2 flops each: 4 * sum(L) * Hq * d
     (the attention term 4BSd of Eq. (flops-layer), per query head)."""
     return 4 * int(np.asarray(seq_lens, dtype=np.int64).sum()) * num_q_heads * head_dim
+
+
+def prefill_flops(seq_lens, q_lens, num_q_heads: int, head_dim: int) -> int:
+    """Causal chunked prefill: query i of a sequence with L cached tokens,
+    the last Q of them new, sees L - Q + i + 1 keys; each key costs a
+    Q.K^T and a P.V multiply-add per head dimension (4 flops).  Summed over
+    a sequence: Q (L - Q) + Q (Q + 1) / 2 query-key pairs per query head."""
+    L = np.asarray(seq_lens, dtype=np.int64)
+    Q = np.asarray(q_lens, dtype=np.int64)
+    pairs = Q * (L - Q) + Q * (Q + 1) // 2
+    return 4 * int(pairs.sum()) * num_q_heads * head_dim
+
+
+def prefill_bytes(seq_lens, q_lens, num_q_heads: int, num_kv_heads: int, head_dim: int,
+                  elem_bytes: int = 2) -> int:
+    """Compulsory HBM bytes of one prefill call: each sequence's K/V once,
+    the queries and the outputs."""
+    L = np.asarray(seq_lens, dtype=np.int64)
+    T = int(np.asarray(q_lens, dtype=np.int64).sum())
+    return int(L.sum()) * kv_bytes_per_token(num_kv_heads, head_dim, elem_bytes) + \
+        2 * T * num_q_heads * head_dim * elem_bytes

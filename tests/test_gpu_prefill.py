@@ -1,0 +1,202 @@
+"""GPU parity of the tcgen05 chunked-prefill path against the fp64 oracle.
+
+Tolerance as for decode: max |gpu - oracle| <= 8e-3 (plus the bf16 output
+rounding 2^-8 |ref| on custom edge cases, whose short contexts give large
+outputs) and mean <= 1e-3, every output finite.  The full-size workload
+compares sampled query rows: causal prefill row i of a sequence is decode
+attention over the first p + 1 = L - Q + i + 1 tokens, which the decode
+oracle computes row by row.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_21719_gb300 import inputs
+
+pytestmark = pytest.mark.gpu
+
+MAX_ABS = 8e-3
+MEAN_ABS = 1e-3
+BF16_REL = 2.0 ** -8
+
+
+@pytest.fixture(scope="module")
+def psd():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2608_21719_gb300 import build
+    build.build()
+    from paper_2608_21719_gb300 import ps_decode
+    return ps_decode
+
+
+def _oracle(wl):
+    return oracle.prefill_attention(inputs.bf16_bits(wl.q), inputs.bf16_bits(wl.k_cache),
+                                    inputs.bf16_bits(wl.v_cache), wl.block_table.cpu().numpy(), wl.lengths,
+                                    wl.q_start.cpu().numpy(), wl.k_cache.shape[1], wl.scale)
+
+
+def _gpu(psd, wl, out=None):
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    out = psd.prefill_attention(wl.q, wl.k_cache, wl.v_cache, wl.block_table, wl.seq_lens, wl.q_start,
+                                wl.max_q_len, out=out, scale=wl.scale, device_status=status)
+    torch.cuda.synchronize()
+    return out, int(status.item())
+
+
+def _compare(got, ref, what="", rel=BF16_REL):
+    got = got.float().cpu().numpy().astype(np.float64)
+    assert np.all(np.isfinite(got)), "non-finite output %s" % what
+    err = np.abs(got - ref)
+    excess = err - (MAX_ABS + rel * np.abs(ref))
+    assert excess.max() <= 0, "%s max abs err %.3g (at |ref| %.3g)" % (
+        what, err.max(), np.abs(ref).flat[int(np.argmax(excess))])
+    assert err.mean() <= MEAN_ABS, "%s mean abs err %.3g" % (what, err.mean())
+
+
+def test_tiny_prefill_full_parity(psd):
+    wl = inputs.make_prefill_workload("p1", device="cpu", spare_blocks=4).to("cuda")
+    out, status = _gpu(psd, wl)
+    assert status == 0
+    _compare(out, _oracle(wl), "p1", rel=0.0)
+
+
+# (new tokens, prior tokens) per sequence: one-token chunks, whole prompts,
+# chunks that end exactly on / just past a 128-key tile, ragged query tiles,
+# and an empty chunk.
+EDGE_NEW = [1, 1, 31, 32, 33, 128, 129, 300, 0, 77, 256]
+EDGE_PRIOR = [0, 200, 0, 96, 95, 0, 127, 1, 50, 1000, 384]
+
+
+@pytest.mark.parametrize("Hq,Hkv", [(8, 8), (4, 2), (8, 2), (32, 8), (64, 8), (12, 2), (16, 1)])
+@pytest.mark.parametrize("bs", [16, 32, 48])
+def test_prefill_edge_chunks_groups_and_block_sizes(psd, Hq, Hkv, bs):
+    wl = inputs.make_prefill_workload("p1", device="cpu", new=EDGE_NEW, prior=EDGE_PRIOR, num_q_heads=Hq,
+                                      num_kv_heads=Hkv, block_size=bs, spare_blocks=3,
+                                      seed=Hq * 31 + bs).to("cuda")
+    out, status = _gpu(psd, wl)
+    assert status == 0
+    _compare(out, _oracle(wl), "edge Hq=%d Hkv=%d bs=%d" % (Hq, Hkv, bs))
+
+
+def test_prefill_one_token_chunks_match_decode_path(psd):
+    """Q_s = 1 everywhere is a decode step; both kernels must agree with the
+    same oracle on the same inputs."""
+    lens = np.asarray([1, 17, 128, 129, 700, 2048], dtype=np.int32)
+    wl = inputs.make_prefill_workload("p1", device="cpu", new=[1] * len(lens), prior=lens - 1,
+                                      num_q_heads=32, num_kv_heads=8, seed=5).to("cuda")
+    out, status = _gpu(psd, wl)
+    assert status == 0
+    ref = oracle.decode_attention(inputs.bf16_bits(wl.q), inputs.bf16_bits(wl.k_cache),
+                                  inputs.bf16_bits(wl.v_cache), wl.block_table.cpu().numpy(), wl.lengths, 8,
+                                  wl.scale)
+    _compare(out, ref, "Q=1")
+    attn = psd.DecodeAttention(len(lens), 32, 8, 128, 16, wl.block_table.shape[1], wl.k_cache.shape[0])
+    dec = attn(wl.q, wl.k_cache, wl.v_cache, wl.block_table, wl.seq_lens, scale=wl.scale)
+    torch.cuda.synchronize()
+    attn.close()
+    _compare(dec, ref, "decode")
+
+
+def test_prefill_is_deterministic_and_blind_to_block_relabelling(psd):
+    wl = inputs.make_prefill_workload("p1", device="cpu", new=[200, 90], prior=[300, 0], num_q_heads=32,
+                                      num_kv_heads=8, spare_blocks=7, seed=9)
+    g = wl.to("cuda")
+    a, sa = _gpu(psd, g)
+    b, sb = _gpu(psd, g)
+    assert sa == sb == 0
+    assert torch.equal(a, b)
+    # Move every page to another physical block: same bits out.
+    nb = wl.k_cache.shape[0]
+    perm = np.random.default_rng(4).permutation(nb)
+    k2 = torch.empty_like(wl.k_cache)
+    v2 = torch.empty_like(wl.v_cache)
+    k2[perm] = wl.k_cache
+    v2[perm] = wl.v_cache
+    bt = wl.block_table.numpy()
+    bt2 = np.where(bt >= 0, perm[np.maximum(bt, 0)], -1).astype(np.int32)
+    g2 = inputs.PrefillWorkload(cfg=wl.cfg, q=wl.q, k_cache=k2, v_cache=v2, block_table=torch.from_numpy(bt2),
+                                seq_lens=wl.seq_lens, q_start=wl.q_start, q_lens=wl.q_lens, lengths=wl.lengths,
+                                scale=wl.scale).to("cuda")
+    c, sc = _gpu(psd, g2)
+    assert sc == 0
+    assert torch.equal(a, c)
+
+
+def test_prefill_flags_bad_block_and_inconsistent_chunk(psd):
+    wl = inputs.make_prefill_workload("p1", device="cpu", new=[40, 30], prior=[100, 10], num_q_heads=8,
+                                      num_kv_heads=2, seed=3).to("cuda")
+    bt_bad = wl.block_table.clone()
+    bt_bad[0, 2] = wl.k_cache.shape[0] + 5
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    psd.prefill_attention(wl.q, wl.k_cache, wl.v_cache, bt_bad, wl.seq_lens, wl.q_start, wl.max_q_len,
+                          scale=wl.scale, device_status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) & psd.PS_DEVICE_BAD_BLOCK
+    # A chunk longer than its sequence is skipped: its rows stay as they were.
+    sl_bad = wl.seq_lens.clone()
+    sl_bad[1] = 20  # Q_1 = 30 > 20
+    status.zero_()
+    out = torch.full_like(wl.q, 3.0)
+    psd.prefill_attention(wl.q, wl.k_cache, wl.v_cache, wl.block_table, sl_bad, wl.q_start, wl.max_q_len,
+                          out=out, scale=wl.scale, device_status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) & psd.PS_DEVICE_LEN_CLAMPED
+    assert torch.all(out[40:] == 3.0)
+    ref = _oracle(wl)
+    _compare(out[:40], ref[:40], "valid sequence next to a skipped one")
+
+
+def test_prefill_rejects_bad_arguments(psd):
+    wl = inputs.make_prefill_workload("p1", device="cpu", new=[5], prior=[5]).to("cuda")
+    out = torch.empty_like(wl.q)
+    args = [wl.q, wl.k_cache, wl.v_cache, wl.block_table, wl.seq_lens, wl.q_start, out, 1, 5, 5, 8, 2, 128, 16,
+            wl.block_table.shape[1], wl.k_cache.shape[0], wl.scale, None, None]
+    bad_dim = list(args)
+    bad_dim[12] = 64
+    with pytest.raises(psd.PsError):
+        psd.ps_prefill_attention(*bad_dim)
+    bad_group = list(args)
+    bad_group[11] = 3  # 8 q heads over 3 kv heads
+    with pytest.raises(psd.PsError):
+        psd.ps_prefill_attention(*bad_group)
+    bad_bs = list(args)
+    bad_bs[13] = 8
+    with pytest.raises(psd.PsError):
+        psd.ps_prefill_attention(*bad_bs)
+    bad_scale = list(args)
+    bad_scale[16] = float("nan")
+    with pytest.raises(psd.PsError):
+        psd.ps_prefill_attention(*bad_scale)
+    psd.ps_prefill_attention(*args)
+    torch.cuda.synchronize()
+
+
+def test_full_size_prefill_sampled_rows(psd):
+    """The 8-sequence Llama-3-8B chunked-prefill batch at full size, in the
+    launch the bench times; 48 sampled query rows (all heads) per call are
+    checked as decode rows of the truncated context."""
+    wl = inputs.make_prefill_workload("p2", device="cuda")
+    out, status = _gpu(psd, wl)
+    assert status == 0
+    assert torch.isfinite(out.float()).all()
+    rng = np.random.default_rng(12)
+    qs = wl.q_start.cpu().numpy()
+    rows, sl = [], []
+    for s in range(len(wl.lengths)):
+        Q, L = int(wl.q_lens[s]), int(wl.lengths[s])
+        picks = {0, Q - 1} | set(rng.integers(0, Q, size=4).tolist())
+        for i in sorted(picks):
+            rows.append(int(qs[s]) + i)
+            sl.append((s, L - Q + i + 1))
+    bt = wl.block_table.cpu().numpy()
+    k_bits = inputs.bf16_bits(wl.k_cache)
+    v_bits = inputs.bf16_bits(wl.v_cache)
+    q_rows = inputs.bf16_bits(wl.q[rows])
+    ref = oracle.decode_attention(q_rows, k_bits, v_bits, bt[[s for s, _ in sl]],
+                                  np.asarray([l for _, l in sl], dtype=np.int32), wl.k_cache.shape[1], wl.scale)
+    got = out[rows].float().cpu().numpy().astype(np.float64)
+    err = np.abs(got - ref)
+    assert err.max() <= MAX_ABS, err.max()
+    assert err.mean() <= MEAN_ABS, err.mean()
