@@ -38,6 +38,9 @@ if ROOT not in sys.path:
 METRIC = "decode-attention KV-read GB/s & fraction of HBM peak; decode tokens/s (1 GB300)"
 FALLBACK_HBM_GBS = 6800.0
 PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "ps_decode_kernel_llama3-8b-decode.md")
+PREFILL_SUMMARY = os.path.join(ROOT, "profiles", "ps_prefill_kernel_llama3-8b-chunked-prefill.md")
+PREFILL_SOURCE = os.path.join(ROOT, "paper_2608_21719_gb300", "csrc", "ps_prefill.cu")
+FALLBACK_BF16_TFLOPS = 1900.0
 KERNEL_SOURCE = os.path.join(ROOT, "paper_2608_21719_gb300", "csrc", "ps_decode_kernels.cu")
 CLOCK_QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
                "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
@@ -54,6 +57,9 @@ def parse_args(argv=None):
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="CPU time budget of the oracle baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--prefill", action="store_true",
+                    help="time the tcgen05 chunked-prefill attention on the 8-sequence Llama-3-8B "
+                         "prefill batch instead (metric: TFLOP/s)")
     ap.add_argument("--transfer", choices=["pack", "unpack"], default=None,
                     help="time the KV hand-off gather (pack) or scatter (unpack) of the whole batch instead")
     ap.add_argument("--min-stages", type=int, default=0,
@@ -103,12 +109,12 @@ def measured_peaks():
         return FALLBACK_HBM_GBS, "fallback"
 
 
-def profiled_traffic():
-    """Per-launch DRAM bytes of the partial kernel from the committed ncu
-    summary, or None when the kernel source changed since it was taken."""
+def profiled_traffic(summary=PROFILE_SUMMARY, source=KERNEL_SOURCE):
+    """Per-launch DRAM bytes of a kernel from its committed ncu summary, or
+    None when the kernel source changed since it was taken."""
     try:
-        text = open(PROFILE_SUMMARY).read()
-        src_hash = hashlib.sha256(open(KERNEL_SOURCE, "rb").read()).hexdigest()
+        text = open(summary).read()
+        src_hash = hashlib.sha256(open(source, "rb").read()).hexdigest()
     except OSError:
         return None
     vals = {}
@@ -486,6 +492,139 @@ def run_transfer(args):
     }
 
 
+def bf16_peak():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["bf16_tflops"]), "measured"
+    except Exception:
+        return FALLBACK_BF16_TFLOPS, "fallback"
+
+
+def time_prefill_oracle(wl, budget_s, threads):
+    """The prefill oracle on a causal prefix of one sequence's chunk (the
+    first n new tokens, which later tokens cannot influence), n grown until
+    one call takes about budget_s.  Returns (flops/s, description)."""
+    import numpy as np
+
+    import oracle
+    from paper_2608_21719_gb300 import inputs, roofline
+
+    s = int(np.argmax(wl.q_lens))
+    Q, L = int(wl.q_lens[s]), int(wl.lengths[s])
+    prior = L - Q
+    bt = wl.block_table[s:s + 1].cpu().numpy()
+    k_bits = inputs.bf16_bits(wl.k_cache)
+    v_bits = inputs.bf16_bits(wl.v_cache)
+    q0 = int(wl.q_start[s].item())
+    Hkv = wl.k_cache.shape[1]
+    n = 4
+    while True:
+        q_bits = inputs.bf16_bits(wl.q[q0:q0 + n])
+        t0 = time.perf_counter()
+        oracle.prefill_attention(q_bits, k_bits, v_bits, bt, np.asarray([prior + n], dtype=np.int32),
+                                 np.asarray([0, n], dtype=np.int32), Hkv, wl.scale, num_threads=threads)
+        dt = time.perf_counter() - t0
+        fl = roofline.prefill_flops([prior + n], [n], wl.q.shape[1], wl.q.shape[2])
+        if dt >= budget_s or n >= Q:
+            return fl / dt, "sequence %d: first %d of its %d new tokens over %d cached (%.2f GFLOP)" % (
+                s, n, Q, prior, fl / 1e9)
+        n = min(Q, max(n + 1, int(n * min(8.0, 1.3 * budget_s / max(dt, 1e-4)))))
+
+
+def run_prefill(args):
+    """Chunked-prefill attention (tcgen05) over the whole 8-sequence batch;
+    metric: causal attention FLOPs / time."""
+    import torch
+
+    from paper_2608_21719_gb300 import inputs, ps_decode, roofline
+
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+    cfg = inputs.PREFILL_CONFIGS["p2"]
+    wl = inputs.make_prefill_workload(cfg, device=dev)
+    Hq, d = wl.q.shape[1], wl.q.shape[2]
+    flops = roofline.prefill_flops(wl.lengths, wl.q_lens, Hq, d)
+    out = torch.empty_like(wl.q)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    flush_buf = torch.empty(max(2 * l2, 64 << 20) // 4, dtype=torch.int32, device=dev)
+    sink = torch.empty((), dtype=torch.int32, device=dev)
+
+    def step():
+        ps_decode.prefill_attention(wl.q, wl.k_cache, wl.v_cache, wl.block_table, wl.seq_lens, wl.q_start,
+                                    wl.max_q_len, out=out, scale=wl.scale, device_status=status,
+                                    stream=stream.cuda_stream)
+
+    def flush():
+        flush_buf.zero_()
+        torch.amax(flush_buf, dim=0, out=sink)
+
+    for _ in range(max(args.warmup, 3)):
+        flush()
+        step()
+    torch.cuda.synchronize(dev)
+    K = args.steps
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    with ClockSampler(os.environ.get("CUDA_VISIBLE_DEVICES", "0").split(",")[0] or "0") as clk:
+        for a, b in ev:
+            flush()
+            a.record(stream)
+            step()
+            b.record(stream)
+        torch.cuda.synchronize(dev)
+    assert int(status.item()) == 0, "device status %d" % int(status.item())
+    ms = statistics.mean(a.elapsed_time(b) for a, b in ev)
+    tflops = flops / (ms * 1e-3) / 1e12
+
+    # End to end: pinned host Q and metadata in, output back, every step.
+    q_h = wl.q.cpu().pin_memory()
+    meta_h = [t.cpu().pin_memory() for t in (wl.block_table, wl.seq_lens, wl.q_start)]
+    q_d = torch.empty_like(wl.q)
+    meta_d = [torch.empty_like(t) for t in (wl.block_table, wl.seq_lens, wl.q_start)]
+    out_h = torch.empty(out.shape, dtype=out.dtype, pin_memory=True)
+    K2 = max(3, min(K, 50))
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize(dev)
+    e0.record(stream)
+    for _ in range(K2):
+        q_d.copy_(q_h, non_blocking=True)
+        for dst, src in zip(meta_d, meta_h):
+            dst.copy_(src, non_blocking=True)
+        ps_decode.prefill_attention(q_d, wl.k_cache, wl.v_cache, meta_d[0], meta_d[1], meta_d[2], wl.max_q_len,
+                                    out=out, scale=wl.scale, device_status=status, stream=stream.cuda_stream)
+        out_h.copy_(out, non_blocking=True)
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    e2e_ms = e0.elapsed_time(e1) / K2
+    h2d = q_h.numel() * 2 + sum(t.numel() * 4 for t in meta_h)
+    d2h = out_h.numel() * 2
+
+    peak, kind = bf16_peak()
+    line = {
+        "metric": "chunked-prefill attention TFLOP/s (causal, paged KV, tcgen05)", "value": round(tflops, 2),
+        "unit": "TFLOP/s", "n_gpus": 1, "steps": K, "warmup": args.warmup, "ms_per_step": round(ms, 5),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": cfg.name, "num_seqs": cfg.num_seqs, "num_q_heads": Hq,
+                   "num_kv_heads": wl.k_cache.shape[1], "head_dim": d, "block_size": wl.k_cache.shape[2],
+                   "new_tokens": int(wl.q_lens.sum()), "cached_tokens": int(wl.lengths.sum()),
+                   "flops_per_step": flops, "l2": "write-then-read flush before every step"},
+        "roofline": {"kernel": "ps_prefill_kernel", "bound": "tensor", "achieved": round(tflops, 1), "peak": peak,
+                     "peak_kind": kind + " (cuBLAS bf16 burst)", "unit": "TFLOP/s", "frac": round(tflops / peak, 4),
+                     "traffic": profiled_traffic(PREFILL_SUMMARY, PREFILL_SOURCE)},
+        "e2e": {"value": round(flops / (e2e_ms * 1e-3) / 1e12, 2), "unit": "TFLOP/s", "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h},
+        "gpu_launches": K,
+        "clocks": clk.summary(),
+    }
+    if not args.no_cpu_baseline:
+        threads = os.cpu_count() or 1
+        rate, sample = time_prefill_oracle(wl, min(args.cpu_seconds, 20.0), threads)
+        line["cpu_baseline"] = {"value": round(rate / 1e12, 6), "unit": "TFLOP/s", "cores": threads,
+                                "kind": "oracle", "sample": sample}
+    return line
+
+
 # ------------------------------------------------------- reference arm ------
 
 def run_reference(args):
@@ -536,6 +675,8 @@ def main(argv=None):
     args = parse_args(argv)
     if args.impl == "reference":
         line = run_reference(args)
+    elif args.prefill:
+        line = run_prefill(args)
     elif args.transfer:
         line = run_transfer(args)
     else:

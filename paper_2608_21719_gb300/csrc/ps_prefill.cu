@@ -11,12 +11,15 @@
 // Tiling.  One CTA per (KV head j, sequence s, query tile).  A query tile is
 // 128 MMA rows: 128 / g consecutive query tokens times the g query heads of
 // group j (row = token * g + head), so every K/V tile staged in shared memory
-// serves the whole group.  Keys stream in tiles of 128 through a two-stage
-// ring; every 16-key chunk of a tile is one TMA box of a (block, kv-head) page
+// serves the whole group.  Keys stream in tiles of 128 through shared-memory
+// rings; every 16-key chunk of a tile is one TMA box of a (block, kv-head) page
 // of the cache, addressed through the block table.
 //
-// Per key tile n (warp roles, 6 warps):
-//   warp 0     TMA producer: Q once, then K_n and V_n into the stage ring.
+// Per key tile n (warp roles, 7 warps):
+//   warps 0, 6 TMA producers: Q once and K_n into a three-stage ring (warp 0),
+//              V_n into a two-stage ring (warp 6).  A K stage is released as
+//              soon as its Q K^T has run, so keys are fetched further ahead
+//              than values, which are held until their P V has run.
 //   warp 1     MMA issuer (one thread): S_n = Q K_n^T into one of two TMEM
 //              score buffers (M = 128, N = 128, K = 128), then, once the
 //              softmax has written P_{n-1}, O += P_{n-1} V_{n-1} into the
@@ -53,13 +56,15 @@ constexpr int kD = 128;            // head_dim
 constexpr int kRows = 128;         // MMA M: query rows per tile
 constexpr int kKeys = 128;         // MMA N of S, K of P.V: keys per tile
 constexpr int kChunk = 16;         // keys per TMA box (one page slice)
-constexpr int kThreads = 192;
+constexpr int kKStages = 3;         // K ring: a stage is free once its Q K^T is done
+constexpr int kVStages = 2;         // V ring: a stage is free once its P V is done
+constexpr int kThreads = 224;
 constexpr int kHalf = kRows * 64 * 2;   // one 64-column half of a 128-row tile: 16 KiB
 constexpr int kTile = 2 * kHalf;        // 32 KiB
 constexpr int kOffQ = 0;
-constexpr int kOffK = kOffQ + kTile;    // two stages
-constexpr int kOffV = kOffK + 2 * kTile;
-constexpr int kOffP = kOffV + 2 * kTile;
+constexpr int kOffK = kOffQ + kTile;
+constexpr int kOffV = kOffK + kKStages * kTile;
+constexpr int kOffP = kOffV + kVStages * kTile;
 constexpr int kOffBar = kOffP + kTile;
 constexpr int kSmemBytes = 1024 + kOffBar + 256;  // 1 KiB of alignment slack
 constexpr uint32_t kTmemCols = 512;
@@ -253,21 +258,27 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     uint64_t *bars = reinterpret_cast<uint64_t *>(sm + kOffBar);
     const uint32_t bar_q = saddr(bars + 0);
-    auto bar_kfull = [&](int st) { return saddr(bars + 1 + st); };
-    auto bar_vfull = [&](int st) { return saddr(bars + 3 + st); };
-    auto bar_kvfree = [&](int st) { return saddr(bars + 5 + st); };
-    auto bar_sfull = [&](int b) { return saddr(bars + 7 + b); };
-    auto bar_sfree = [&](int b) { return saddr(bars + 9 + b); };
-    const uint32_t bar_pfull = saddr(bars + 11), bar_odone = saddr(bars + 12), bar_mma_end = saddr(bars + 13);
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + 14);
-    volatile int *abort = reinterpret_cast<volatile int *>(bars + 15);
+    auto bar_kfull = [&](int st) { return saddr(bars + 1 + st); };   // [kKStages]
+    auto bar_kfree = [&](int st) { return saddr(bars + 4 + st); };   // [kKStages]
+    auto bar_vfull = [&](int st) { return saddr(bars + 7 + st); };   // [kVStages]
+    auto bar_vfree = [&](int st) { return saddr(bars + 9 + st); };   // [kVStages]
+    auto bar_sfull = [&](int b) { return saddr(bars + 11 + b); };
+    auto bar_sfree = [&](int b) { return saddr(bars + 13 + b); };
+    const uint32_t bar_pfull = saddr(bars + 15), bar_odone = saddr(bars + 16), bar_mma_end = saddr(bars + 17);
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + 18);
+    volatile int *abort = reinterpret_cast<volatile int *>(bars + 19);
 
     if (tid == 0) {
         mbar_init(bar_q, 1);
-        for (int i = 0; i < 2; ++i) {
+        for (int i = 0; i < kKStages; ++i) {
             mbar_init(bar_kfull(i), 1);
+            mbar_init(bar_kfree(i), 1);
+        }
+        for (int i = 0; i < kVStages; ++i) {
             mbar_init(bar_vfull(i), 1);
-            mbar_init(bar_kvfree(i), 1);
+            mbar_init(bar_vfree(i), 1);
+        }
+        for (int i = 0; i < 2; ++i) {
             mbar_init(bar_sfull(i), 1);
             mbar_init(bar_sfree(i), 4);
         }
@@ -290,49 +301,50 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     const uint32_t sQ = saddr(sm + kOffQ), sK = saddr(sm + kOffK), sV = saddr(sm + kOffV), sP = saddr(sm + kOffP);
 
-    if (warp == 0) {
-        // ------------------------------------------------------ producer --
-        if (lane == 0) {
+    if (warp == 0 || warp == 6) {
+        // ----------------------------------------------------- producers --
+        const bool is_k = warp == 0;
+        if (is_k && lane == 0) {
             asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmQ)) : "memory");
             asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
-            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
             mbar_expect_tx(bar_q, (uint32_t)(2 * 128 * g * tpt));
             tma_load_3d(sQ, &tmQ, 0, j * g, qs0 + tok0, bar_q);
             tma_load_3d(sQ + kHalf, &tmQ, 64, j * g, qs0 + tok0, bar_q);
         }
+        if (!is_k && lane == 0)
+            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
+        const int stages = is_k ? kKStages : kVStages;
+        const uint32_t ring = is_k ? sK : sV;
+        const CUtensorMap *tm = is_k ? &tmK : &tmV;
         const int *bt_row = p.block_table + (size_t)s * p.max_blocks_per_seq;
-        const int tensor = lane >> 4, half = (lane >> 3) & 1, c = lane & 7;
-        const CUtensorMap *tm = tensor ? &tmV : &tmK;
+        const int half = (lane >> 3) & 1, c = lane & 7;  // lanes 0-15: 8 chunks x 2 halves
         int issued = 0;
         for (int n = 0; n < ntiles; ++n) {
-            const int st = n & 1;
-            if (n >= 2 && !warp_wait(bar_kvfree(st), ((n >> 1) - 1) & 1, abort, p.status)) break;
+            const int st = n % stages, use = n / stages;
+            if (n >= stages &&
+                !warp_wait(is_k ? bar_kfree(st) : bar_vfree(st), (use - 1) & 1, abort, p.status))
+                break;
             const int base = n * kKeys;
             const int nc = (min(kKeys, kv_limit - base) + kChunk - 1) / kChunk;
-            if (lane == 0) {
-                mbar_expect_tx(bar_kfull(st), (uint32_t)(nc * 2 * kChunk * 128));
-                mbar_expect_tx(bar_vfull(st), (uint32_t)(nc * 2 * kChunk * 128));
-            }
+            const uint32_t full = is_k ? bar_kfull(st) : bar_vfull(st);
+            if (lane == 0) mbar_expect_tx(full, (uint32_t)(nc * 2 * kChunk * 128));
             __syncwarp();
-            if (c < nc) {
+            if (lane < 16 && c < nc) {
                 const int t0 = base + c * kChunk;
                 const int lb = t0 / p.block_size;
                 const int b = __ldg(bt_row + lb);
                 int page = -1;  // out of range: TMA fills zeros
                 if (b >= 0 && (long long)b < p.num_blocks) page = b * p.num_kv_heads + j;
-                else if (p.status) atomicOr(p.status, (unsigned)PS_DEVICE_BAD_BLOCK);
-                const uint32_t dst = (tensor ? sV : sK) + st * kTile + half * kHalf + c * (kChunk * 128);
-                tma_load_3d(dst, tm, half * 64, t0 - lb * p.block_size, page,
-                            tensor ? bar_vfull(st) : bar_kfull(st));
+                else if (p.status && is_k) atomicOr(p.status, (unsigned)PS_DEVICE_BAD_BLOCK);
+                tma_load_3d(ring + st * kTile + half * kHalf + c * (kChunk * 128), tm, half * 64,
+                            t0 - lb * p.block_size, page, full);
             }
             issued = n + 1;
         }
         // Drain: the last copies of each stage must land before the CTA exits.
-        for (int n = max(0, issued - 2); n < issued; ++n) {
-            drain_phase(bar_kfull(n & 1), (n >> 1) & 1);
-            drain_phase(bar_vfull(n & 1), (n >> 1) & 1);
-        }
-        drain_phase(bar_q, 0);
+        for (int n = max(0, issued - stages); n < issued; ++n)
+            drain_phase(is_k ? bar_kfull(n % stages) : bar_vfull(n % stages), (n / stages) & 1);
+        if (is_k) drain_phase(bar_q, 0);
     } else if (warp == 1) {
         // ---------------------------------------------------- MMA issuer --
         constexpr uint32_t idS = instr_desc(kRows, kKeys, 0);
@@ -340,8 +352,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         bool ok = warp_wait(bar_q, 0, abort, p.status);
         for (int n = 0; ok && n <= ntiles; ++n) {
             if (n < ntiles) {
-                const int st = n & 1, b = n & 1;
-                if (!warp_wait(bar_kfull(st), (n >> 1) & 1, abort, p.status)) { ok = false; break; }
+                const int st = n % kKStages, b = n & 1;
+                if (!warp_wait(bar_kfull(st), (n / kKStages) & 1, abort, p.status)) { ok = false; break; }
                 if (n >= 2 && !warp_wait(bar_sfree(b), ((n >> 1) - 1) & 1, abort, p.status)) { ok = false; break; }
                 tc_fence_after();
                 if (lane == 0) {
@@ -353,12 +365,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                              kk > 0);
                     }
                     umma_commit(bar_sfull(b));
+                    umma_commit(bar_kfree(st));
                 }
                 __syncwarp();
             }
             if (n >= 1) {
-                const int m = n - 1, st = m & 1;
-                if (!warp_wait(bar_vfull(st), (m >> 1) & 1, abort, p.status)) { ok = false; break; }
+                const int m = n - 1, st = m % kVStages;
+                if (!warp_wait(bar_vfull(st), (m / kVStages) & 1, abort, p.status)) { ok = false; break; }
                 const uint32_t vb = sV + st * kTile;
                 const int valid = kv_limit - m * kKeys;
                 if (valid < kKeys) {
@@ -382,7 +395,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                              smem_desc(vb + kk * 2048, 16384, 1024), idO, (m > 0 || kk > 0) ? 1u : 0u);
                     }
                     umma_commit(bar_odone);
-                    umma_commit(bar_kvfree(st));
+                    umma_commit(bar_vfree(st));
                 }
                 __syncwarp();
             }
