@@ -8,7 +8,7 @@
 // has L_s cached tokens whose last Q_s are the new (query) tokens; query i sits
 // at position p = L_s - Q_s + i and sees keys 0 .. p.
 //
-// Tiling.  One CTA per (KV head j, sequence s, query tile).  A query tile is
+// Tiling.  One CTA per (query tile, KV head j, sequence s).  A query tile is
 // 128 MMA rows: 128 / g consecutive query tokens times the g query heads of
 // group j (row = token * g + head), so every K/V tile staged in shared memory
 // serves the whole group.  Keys stream in tiles of 128 through shared-memory
@@ -237,8 +237,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int j = blockIdx.x, s = blockIdx.y;
-    const int qt = p.num_qtiles - 1 - (int)blockIdx.z;  // heaviest (last) query tiles first
+    // Consecutive CTAs share a (sequence, KV head), heaviest (last) query
+    // tile first: the few K/V streams in flight at a time stay in L2.
+    const int qt = p.num_qtiles - 1 - (int)blockIdx.x;
+    const int j = blockIdx.y, s = blockIdx.z;
     const int g = p.group, tpt = p.tokens_per_tile;
 
     // Sequence geometry (uniform over the CTA).
@@ -603,7 +605,7 @@ extern "C" ps_status_t ps_prefill_attention(const void *q, const void *k_cache, 
     pp.max_blocks_per_seq = max_blocks_per_seq;
     pp.num_blocks = num_blocks;
     pp.scale_log2 = scale * 1.4426950408889634f;
-    const dim3 grid((unsigned)num_kv_heads, (unsigned)num_seqs, (unsigned)nqt);
+    const dim3 grid((unsigned)nqt, (unsigned)num_kv_heads, (unsigned)num_seqs);
     ps_prefill_kernel<<<grid, kThreads, kSmemBytes, reinterpret_cast<cudaStream_t>(stream)>>>(tmQ, tmK, tmV, pp);
     return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
 }
