@@ -37,6 +37,9 @@ if ROOT not in sys.path:
 
 METRIC = "decode-attention KV-read GB/s & fraction of HBM peak; decode tokens/s (1 GB300)"
 FALLBACK_HBM_GBS = 6800.0
+NOMINAL_HBM_GBS = 7900.0  # NVIDIA's GB300 HBM3e figure, for a labelled second fraction only
+# Layers of the model each workload is shaped after (8B: 32, 32B: 64, 70B: 80).
+MODEL_LAYERS = {1: None, 2: 32, 3: 32, 4: 64, 5: 80}
 PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "ps_decode_kernel_llama3-8b-decode.md")
 PREFILL_SUMMARY = os.path.join(ROOT, "profiles", "ps_prefill_kernel_llama3-8b-chunked-prefill.md")
 PREFILL_SOURCE = os.path.join(ROOT, "paper_2608_21719_gb300", "csrc", "ps_prefill.cu")
@@ -390,8 +393,15 @@ def run_ours(args):
         },
         "frac_of_hbm_peak": round(alg["total"] / (ms_per_step * 1e-3) / 1e9 / hbm_peak, 4),
         "decode_tokens_per_s": round(wl.num_seqs * world * K / (total_ms * 1e-3), 1),
-        "kernel_ms": {"mean": round(ms_per_step, 5), "min": round(min(step_ms), 5),
-                      "max": round(max(step_ms), 5)},
+        # Context only: one attention call per layer, so a whole model's
+        # decode step over this batch needs n_layers of them.
+        "attention_only_tokens_per_s": (
+            None if MODEL_LAYERS.get(args.config) is None else
+            {"n_layers": MODEL_LAYERS[args.config],
+             "value": round(wl.num_seqs * world * K / (total_ms * 1e-3) / MODEL_LAYERS[args.config], 1)}),
+        "kernel_ms": {"mean": round(ms_per_step, 5), "median": round(statistics.median(step_ms), 5),
+                      "min": round(min(step_ms), 5), "max": round(max(step_ms), 5)},
+        "frac_of_nominal_hbm": round(alg["total"] / (ms_per_step * 1e-3) / 1e9 / NOMINAL_HBM_GBS, 4),
         "roofline": {
             "kernel": "ps_decode_kernel",
             "bound": "hbm",
