@@ -478,6 +478,7 @@ def run_transfer(args):
     torch.cuda.synchronize(dev)
     K = args.steps
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    launches0 = ps_decode.ps_decode_launch_count()
     with ClockSampler(os.environ.get("CUDA_VISIBLE_DEVICES", "0").split(",")[0] or "0") as clk:
         for a, b in ev:
             flush_buf.zero_(); torch.amax(flush_buf, dim=0, out=sink)
@@ -485,6 +486,7 @@ def run_transfer(args):
             step()
             b.record(stream)
         torch.cuda.synchronize(dev)
+    launches = ps_decode.ps_decode_launch_count() - launches0
     assert int(status.item()) == 0
     ms = statistics.mean(a.elapsed_time(b) for a, b in ev)
     moved = 2 * int(sizes.sum()) * 2  # every element read once and written once
@@ -498,6 +500,7 @@ def run_transfer(args):
         "roofline": {"kernel": "ps_kv_transfer_kernel", "bound": "hbm", "achieved": round(gbs, 1), "peak": peak,
                      "peak_kind": kind + " (copy bandwidth)", "unit": "GB/s", "frac": round(gbs / peak, 4),
                      "traffic": None},
+        "gpu_launches": launches,
         "clocks": clk.summary(),
     }
 
@@ -576,6 +579,7 @@ def run_prefill(args):
     torch.cuda.synchronize(dev)
     K = args.steps
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    launches0 = ps_decode.ps_decode_launch_count()
     with ClockSampler(os.environ.get("CUDA_VISIBLE_DEVICES", "0").split(",")[0] or "0") as clk:
         for a, b in ev:
             flush()
@@ -583,6 +587,7 @@ def run_prefill(args):
             step()
             b.record(stream)
         torch.cuda.synchronize(dev)
+    launches = ps_decode.ps_decode_launch_count() - launches0
     assert int(status.item()) == 0, "device status %d" % int(status.item())
     ms = statistics.mean(a.elapsed_time(b) for a, b in ev)
     tflops = flops / (ms * 1e-3) / 1e12
@@ -624,7 +629,7 @@ def run_prefill(args):
                      "traffic": profiled_traffic(PREFILL_SUMMARY, PREFILL_SOURCE)},
         "e2e": {"value": round(flops / (e2e_ms * 1e-3) / 1e12, 2), "unit": "TFLOP/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
-        "gpu_launches": K,
+        "gpu_launches": launches,
         "clocks": clk.summary(),
     }
     if not args.no_cpu_baseline:

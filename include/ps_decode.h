@@ -319,7 +319,9 @@ ps_status_t ps_decode_attention_noalloc(const void *q, const void *k_cache, cons
                                         int block_size, int max_blocks_per_seq, long long num_blocks,
                                         float scale, void *stream);
 
-/* Number of kernels this library has launched in this process. */
+/* Number of kernels this library has launched in this process through the
+ * decode, fused-append, prefill and KV hand-off entry points (the
+ * workspace-free entry point is not counted). */
 unsigned long long ps_decode_launch_count(void);
 
 /* Static description of a status code. */

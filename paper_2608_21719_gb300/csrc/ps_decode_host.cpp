@@ -162,6 +162,8 @@ ps_status_t run_planned(ps_decode_plan *p, const void *q, const void *k, const v
 
 }  // namespace
 
+void ps::note_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
+
 extern "C" {
 
 ps_status_t ps_decode_plan_create_ex(int num_seqs, int num_q_heads, int num_kv_heads, int head_dim, int block_size,

@@ -98,6 +98,9 @@ struct DecodeParams {
 };
 
 // Launcher (ps_decode_kernels.cu).  Returns cudaSuccess or the launch error.
+// Adds one to the library's launch counter (ps_decode_launch_count()).
+void note_launch();
+
 cudaError_t launch_decode(const DecodeParams &p, const CUtensorMap &tmK, const CUtensorMap &tmV, int grid_ctas,
                           size_t smem_bytes, cudaStream_t stream);
 

@@ -168,7 +168,9 @@ ps_status_t launch_xfer(const XferParams &xp, void *stream) {
             cudaSuccess)
         return PS_ERR_CUDA;
     ps_kv_transfer_kernel<kPack><<<sms * kXferCtasPerSm, kXferWarps * 32, smem, reinterpret_cast<cudaStream_t>(stream)>>>(xp);
-    return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
+    if (cudaGetLastError() != cudaSuccess) return PS_ERR_CUDA;
+    ps::note_launch();
+    return PS_OK;
 }
 
 }  // namespace

@@ -49,6 +49,7 @@
 #include <mutex>
 
 #include "ps_decode.h"
+#include "ps_internal.h"
 
 namespace {
 
@@ -607,5 +608,7 @@ extern "C" ps_status_t ps_prefill_attention(const void *q, const void *k_cache, 
     pp.scale_log2 = scale * 1.4426950408889634f;
     const dim3 grid((unsigned)nqt, (unsigned)num_kv_heads, (unsigned)num_seqs);
     ps_prefill_kernel<<<grid, kThreads, kSmemBytes, reinterpret_cast<cudaStream_t>(stream)>>>(tmQ, tmK, tmV, pp);
-    return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
+    if (cudaGetLastError() != cudaSuccess) return PS_ERR_CUDA;
+    ps::note_launch();
+    return PS_OK;
 }
