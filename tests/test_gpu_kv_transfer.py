@@ -76,6 +76,8 @@ def test_bad_block_is_skipped_and_flagged(psd):
     off = torch.from_numpy(oracle.packed_offsets(L, Hkv, 128)).cuda()
     dst = torch.zeros(int(2 * Hkv * L.sum() * 128), dtype=torch.int16, device="cuda")
     status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    before = psd.ps_decode_launch_count()
     psd.ps_kv_pack(wl.k_cache, wl.v_cache, bt_bad, 4, wl.seq_lens, 2, Hkv, 128, bs, nb, off, dst, status, None)
     torch.cuda.synchronize()
+    assert psd.ps_decode_launch_count() - before == 1
     assert int(status.item()) & psd.PS_DEVICE_BAD_BLOCK

@@ -200,3 +200,11 @@ def test_full_size_prefill_sampled_rows(psd):
     err = np.abs(got - ref)
     assert err.max() <= MAX_ABS, err.max()
     assert err.mean() <= MEAN_ABS, err.mean()
+
+
+def test_prefill_counts_one_launch_per_call(psd):
+    wl = inputs.make_prefill_workload("p1", device="cpu", new=[50, 20], prior=[10, 300]).to("cuda")
+    before = psd.ps_decode_launch_count()
+    _gpu(psd, wl)
+    _gpu(psd, wl)
+    assert psd.ps_decode_launch_count() - before == 2
