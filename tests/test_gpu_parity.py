@@ -108,6 +108,35 @@ def test_forced_splits(psd, max_workers, min_stages):
     _compare(out, _oracle(wl), "split %s/%s" % (max_workers, min_stages))
 
 
+def test_maximum_number_of_sequences(psd):
+    """4096 sequences (the limit of the per-CTA length tables), ragged and
+    partly empty, all compared with the oracle."""
+    lens = np.random.default_rng(41).integers(0, 48, size=4096)
+    lens[::97] = 0
+    wl = _custom(8, 2, 16, lens, seed=41)
+    out, status, _ = _gpu(psd, wl)
+    assert status == 0
+    _compare(out, _oracle(wl), "S=4096")
+    assert torch.all(out[torch.from_numpy(np.nonzero(lens == 0)[0]).cuda()] == 0)
+
+
+def test_largest_block_size(psd):
+    wl = _custom(8, 2, 256, [1, 255, 256, 257, 1000, 5000, 0, 4096], seed=42)
+    out, status, _ = _gpu(psd, wl)
+    assert status == 0
+    _compare(out, _oracle(wl), "bs=256")
+
+
+def test_one_long_sequence_split_over_every_worker(psd):
+    """A single 131072-token context: its one segment per KV head is cut into
+    a piece per streaming warp and merged by the last arriving warp."""
+    wl = _custom(8, 1, 16, [131072], seed=43, spare=2)
+    out, status, info = _gpu(psd, wl)
+    assert status == 0
+    assert info["max_workers"] >= 1000
+    _compare(out, _oracle(wl), "L=131072")
+
+
 def test_repeated_calls_reuse_the_workspace_state(psd):
     # Segment counters return to zero after every call; a later call must
     # not see an earlier call's state, and the split is bit-deterministic.

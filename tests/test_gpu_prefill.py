@@ -208,3 +208,20 @@ def test_prefill_counts_one_launch_per_call(psd):
     _gpu(psd, wl)
     _gpu(psd, wl)
     assert psd.ps_decode_launch_count() - before == 2
+
+
+def test_long_prompt_chunk_sampled_rows(psd):
+    """One 8192-token chunk over 4096 cached tokens (128 query tiles of
+    Llama-3-8B heads), checked on sampled rows as decode rows of the
+    truncated context."""
+    wl = inputs.make_prefill_workload("p2", device="cuda", new=[8192], prior=[4096])
+    out, status = _gpu(psd, wl)
+    assert status == 0
+    rows = sorted({0, 1, 31, 32, 4095, 8191} | set(np.random.default_rng(3).integers(0, 8192, size=10).tolist()))
+    ref = oracle.decode_attention(inputs.bf16_bits(wl.q[rows]), inputs.bf16_bits(wl.k_cache), inputs.bf16_bits(wl.v_cache),
+                                  wl.block_table.cpu().numpy()[[0] * len(rows)],
+                                  np.asarray([4096 + i + 1 for i in rows], dtype=np.int32), wl.k_cache.shape[1], wl.scale)
+    got = out[rows].float().cpu().numpy().astype(np.float64)
+    err = np.abs(got - ref)
+    assert err.max() <= MAX_ABS, err.max()
+    assert err.mean() <= MEAN_ABS, err.mean()
