@@ -17,19 +17,21 @@
 //
 // Per key tile n (warp roles, 7 warps):
 //   warps 0, 6 TMA producers: Q once and K_n into a three-stage ring (warp 0),
-//              V_n into a two-stage ring (warp 6).  A K stage is released as
-//              soon as its Q K^T has run, so keys are fetched further ahead
-//              than values, which are held until their P V has run.
+//              V_n into a three-stage ring (warp 6).  A K stage is released
+//              as soon as its Q K^T has run, a V stage once its P V has run.
 //   warp 1     MMA issuer (one thread): S_n = Q K_n^T into one of two TMEM
 //              score buffers (M = 128, N = 128, K = 128), then, once the
-//              softmax has written P_{n-1}, O += P_{n-1} V_{n-1} into the
-//              TMEM output accumulator.  Completion is signalled with
+//              softmax has written P_{n-1}, O += P_{n-1} V_{n-1} with P read
+//              from TMEM and V (MN-major) from shared memory, into the TMEM
+//              output accumulator.  Completion is signalled with
 //              tcgen05.commit on mbarriers.
 //   warps 2-5  softmax, one TMEM lane (= one row) per thread: load the score
 //              row, mask it causally, update the running max m and sum l in
 //              fp32 (base 2, log2 e folded into the scale), write the bf16
-//              probabilities P as the next MMA's A operand, and rescale the
-//              output row in TMEM when the max has grown.
+//              probabilities into TMEM P buffer n & 1 (the A operand of the
+//              P V MMA), and rescale the output row in TMEM when the max has
+//              grown.  Only that rescale waits for the previous P V, so the
+//              exponentials of tile n+1 overlap the P V of tile n.
 // The rescale is lazy: the reference max m only moves when the tile max
 // exceeds it by more than 2^8, so P <= 256 and no value leaves fp32/bf16
 // range; the final O / l is the same quotient whichever reference max was
@@ -58,18 +60,19 @@ constexpr int kRows = 128;         // MMA M: query rows per tile
 constexpr int kKeys = 128;         // MMA N of S, K of P.V: keys per tile
 constexpr int kChunk = 16;         // keys per TMA box (one page slice)
 constexpr int kKStages = 3;         // K ring: a stage is free once its Q K^T is done
-constexpr int kVStages = 2;         // V ring: a stage is free once its P V is done
+constexpr int kVStages = 3;         // V ring: a stage is free once its P V is done
 constexpr int kThreads = 224;
 constexpr int kHalf = kRows * 64 * 2;   // one 64-column half of a 128-row tile: 16 KiB
 constexpr int kTile = 2 * kHalf;        // 32 KiB
 constexpr int kOffQ = 0;
 constexpr int kOffK = kOffQ + kTile;
 constexpr int kOffV = kOffK + kKStages * kTile;
-constexpr int kOffP = kOffV + kVStages * kTile;
-constexpr int kOffBar = kOffP + kTile;
+constexpr int kOffBar = kOffV + kVStages * kTile;
 constexpr int kSmemBytes = 1024 + kOffBar + 256;  // 1 KiB of alignment slack
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kColO = 256;          // S buffers at columns 0 and 128
+// TMEM columns: S buffers at 0 and 128, O at 256, two P buffers (bf16 pairs
+// packed in 32-bit columns, 64 columns each) at 384 and 448.
+constexpr uint32_t kColO = 256, kColP = 384;
 constexpr float kRescaleLog2 = 8.0f;
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;
 
@@ -149,6 +152,15 @@ __device__ __forceinline__ void umma(uint32_t d_tmem, uint64_t a, uint64_t b, ui
         "l"(a), "l"(b), "r"(idesc), "r"(acc)
         : "memory");
 }
+// The same with A read from tensor memory (row = TMEM lane, K packed in bf16
+// pairs along the columns: a K step of 16 is 8 columns).
+__device__ __forceinline__ void umma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b, uint32_t idesc, uint32_t acc) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "r"(a_tmem), "l"(b), "r"(idesc), "r"(acc)
+        : "memory");
+}
 __device__ __forceinline__ void umma_commit(uint32_t bar) {
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
                  : "memory");
@@ -165,6 +177,13 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float *v) {
         : "r"(taddr));
 #pragma unroll
     for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+__device__ __forceinline__ void tmem_st16u(uint32_t taddr, const uint32_t (&v)[16]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(taddr),
+        "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]), "r"(v[9]),
+        "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
+        : "memory");
 }
 __device__ __forceinline__ void tmem_st32(uint32_t taddr, const float (&v)[32]) {
     asm volatile(
@@ -228,9 +247,6 @@ __device__ __forceinline__ void drain_phase(uint32_t bar, uint32_t parity) {
         if (global_ns() - t0 > kWaitLimitNs) return;
 }
 
-// Byte offset of 16-byte chunk c (0..7) of row r in a 128-byte-swizzled
-// [rows][64] half tile.
-__device__ __forceinline__ uint32_t sw128(int r, int c) { return (uint32_t)(r * 128 + ((c ^ (r & 7)) << 4)); }
 
 __global__ void __launch_bounds__(kThreads, 1)
     ps_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
@@ -261,15 +277,19 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     uint64_t *bars = reinterpret_cast<uint64_t *>(sm + kOffBar);
     const uint32_t bar_q = saddr(bars + 0);
-    auto bar_kfull = [&](int st) { return saddr(bars + 1 + st); };   // [kKStages]
-    auto bar_kfree = [&](int st) { return saddr(bars + 4 + st); };   // [kKStages]
-    auto bar_vfull = [&](int st) { return saddr(bars + 7 + st); };   // [kVStages]
-    auto bar_vfree = [&](int st) { return saddr(bars + 9 + st); };   // [kVStages]
-    auto bar_sfull = [&](int b) { return saddr(bars + 11 + b); };
-    auto bar_sfree = [&](int b) { return saddr(bars + 13 + b); };
-    const uint32_t bar_pfull = saddr(bars + 15), bar_odone = saddr(bars + 16), bar_mma_end = saddr(bars + 17);
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + 18);
-    volatile int *abort = reinterpret_cast<volatile int *>(bars + 19);
+    auto bar_kfull = [&](int st) { return saddr(bars + 1 + st); };                        // [kKStages]
+    auto bar_kfree = [&](int st) { return saddr(bars + 1 + kKStages + st); };             // [kKStages]
+    auto bar_vfull = [&](int st) { return saddr(bars + 1 + 2 * kKStages + st); };         // [kVStages]
+    auto bar_vfree = [&](int st) { return saddr(bars + 1 + 2 * kKStages + kVStages + st); };
+    constexpr int kB = 1 + 2 * kKStages + 2 * kVStages;
+    auto bar_sfull = [&](int b) { return saddr(bars + kB + b); };
+    auto bar_sfree = [&](int b) { return saddr(bars + kB + 2 + b); };
+    auto bar_pfull = [&](int b) { return saddr(bars + kB + 4 + b); };
+    auto bar_pfree = [&](int b) { return saddr(bars + kB + 6 + b); };
+    const uint32_t bar_mma_end = saddr(bars + kB + 8);
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + kB + 9);
+    volatile int *abort = reinterpret_cast<volatile int *>(bars + kB + 10);
+    static_assert((1 + 2 * kKStages + 2 * kVStages + 11) * 8 <= 256, "barrier area");
 
     if (tid == 0) {
         mbar_init(bar_q, 1);
@@ -284,9 +304,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int i = 0; i < 2; ++i) {
             mbar_init(bar_sfull(i), 1);
             mbar_init(bar_sfree(i), 4);
+            mbar_init(bar_pfull(i), 128);
+            mbar_init(bar_pfree(i), 1);
         }
-        mbar_init(bar_pfull, 128);
-        mbar_init(bar_odone, 1);
         mbar_init(bar_mma_end, 1);
         *abort = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -302,7 +322,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
-    const uint32_t sQ = saddr(sm + kOffQ), sK = saddr(sm + kOffK), sV = saddr(sm + kOffV), sP = saddr(sm + kOffP);
+    const uint32_t sQ = saddr(sm + kOffQ), sK = saddr(sm + kOffK), sV = saddr(sm + kOffV);
 
     if (warp == 0 || warp == 6) {
         // ----------------------------------------------------- producers --
@@ -389,15 +409,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                     fence_proxy_async_smem();
                     __syncwarp();
                 }
-                if (!warp_wait(bar_pfull, m & 1, abort, p.status)) { ok = false; break; }
+                if (!warp_wait(bar_pfull(m & 1), (m >> 1) & 1, abort, p.status)) { ok = false; break; }
                 tc_fence_after();
                 if (lane == 0) {
+                    const uint32_t pt = tmem + kColP + (m & 1) * (kKeys / 2);
 #pragma unroll
-                    for (int kk = 0; kk < kKeys / 16; ++kk) {
-                        umma(tmem + kColO, smem_desc(sP + (kk >> 2) * kHalf + (kk & 3) * 32, 16, 1024),
-                             smem_desc(vb + kk * 2048, 16384, 1024), idO, (m > 0 || kk > 0) ? 1u : 0u);
-                    }
-                    umma_commit(bar_odone);
+                    for (int kk = 0; kk < kKeys / 16; ++kk)
+                        umma_ts(tmem + kColO, pt + kk * 8, smem_desc(vb + kk * 2048, 16384, 1024), idO,
+                                (m > 0 || kk > 0) ? 1u : 0u);
+                    umma_commit(bar_pfree(m & 1));
                     umma_commit(bar_vfree(st));
                 }
                 __syncwarp();
@@ -440,13 +460,12 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int i = 1; i < kKeys; ++i) mx = fmaxf(mx, sv[i]);
             const float m_tile = mx * sl2;
-            if (n >= 1) {
-                if (!warp_wait(bar_odone, (n - 1) & 1, abort, p.status)) { ok = false; break; }
-                tc_fence_after();
-            }
             const bool grow = m_tile > m_ref + kRescaleLog2;  // always true on the first tile
             const float alpha = grow ? ex2(m_ref - m_tile) : 1.f;
             if (n >= 1 && __any_sync(0xffffffffu, grow)) {
+                // O must hold key tiles 0 .. n-1 before it is rescaled.
+                if (!warp_wait(bar_pfree((n - 1) & 1), ((n - 1) >> 1) & 1, abort, p.status)) { ok = false; break; }
+                tc_fence_after();
 #pragma unroll
                 for (int c = 0; c < 4; ++c) {
                     float ov[32];
@@ -463,27 +482,32 @@ __global__ void __launch_bounds__(kThreads, 1)
                 l *= alpha;
                 m_ref = m_tile;
             }
-            // P row (bf16) as the K-major A operand: [key half][row][64], swizzled.
-            uint8_t *prow = sm + kOffP;
+            // P buffer b was last read by the P V of tile n - 2.
+            if (n >= 2) {
+                if (!warp_wait(bar_pfree(b), ((n >> 1) - 1) & 1, abort, p.status)) { ok = false; break; }
+                tc_fence_after();
+            }
+            // P row (bf16 pairs) into TMEM buffer b, row = this thread's lane:
+            // the A operand of the P V MMA.
 #pragma unroll
-            for (int c = 0; c < 16; ++c) {
-                uint32_t w[4];
+            for (int c = 0; c < 4; ++c) {
+                uint32_t w[16];
 #pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const float a = ex2(fmaf(sv[c * 8 + 2 * e], sl2, -m_ref));
-                    const float bb = ex2(fmaf(sv[c * 8 + 2 * e + 1], sl2, -m_ref));
-                    const __nv_bfloat162 pr = __floats2bfloat162_rn(a, bb);
+                for (int e = 0; e < 16; ++e) {
+                    const int i = c * 32 + 2 * e;
+                    const __nv_bfloat162 pr =
+                        __floats2bfloat162_rn(ex2(fmaf(sv[i], sl2, -m_ref)), ex2(fmaf(sv[i + 1], sl2, -m_ref)));
                     const float2 back = __bfloat1622float2(pr);
                     l += back.x + back.y;
                     w[e] = *reinterpret_cast<const uint32_t *>(&pr);
                 }
-                *reinterpret_cast<uint4 *>(prow + (c >> 3) * kHalf + sw128(r, c & 7)) = make_uint4(w[0], w[1], w[2], w[3]);
+                tmem_st16u(trow + kColP + b * (kKeys / 2) + c * 16, w);
             }
-            fence_proxy_async_smem();
+            tmem_wait_st();
             tc_fence_before();
-            mbar_arrive(bar_pfull);
+            mbar_arrive(bar_pfull(b));
         }
-        if (ok && warp_wait(bar_odone, (ntiles - 1) & 1, abort, p.status)) {
+        if (ok && warp_wait(bar_pfree((ntiles - 1) & 1), ((ntiles - 1) >> 1) & 1, abort, p.status)) {
             tc_fence_after();
             const float inv = 1.f / l;
             uint16_t *orow = p.out + ((size_t)(qs0 + tok0 + tl) * p.num_q_heads + (size_t)j * g + hl) * kD;
