@@ -59,8 +59,14 @@ constexpr int kD = 128;            // head_dim
 constexpr int kRows = 128;         // MMA M: query rows per tile
 constexpr int kKeys = 128;         // MMA N of S, K of P.V: keys per tile
 constexpr int kChunk = 16;         // keys per TMA box (one page slice)
-constexpr int kKStages = 3;         // K ring: a stage is free once its Q K^T is done
-constexpr int kVStages = 3;         // V ring: a stage is free once its P V is done
+#ifndef PS_PREFILL_KSTAGES
+#define PS_PREFILL_KSTAGES 3
+#endif
+#ifndef PS_PREFILL_VSTAGES
+#define PS_PREFILL_VSTAGES 3
+#endif
+constexpr int kKStages = PS_PREFILL_KSTAGES;  // K ring: a stage is free once its Q K^T is done
+constexpr int kVStages = PS_PREFILL_VSTAGES;  // V ring: a stage is free once its P V is done
 constexpr int kThreads = 224;
 constexpr int kHalf = kRows * 64 * 2;   // one 64-column half of a 128-row tile: 16 KiB
 constexpr int kTile = 2 * kHalf;        // 32 KiB
@@ -69,6 +75,7 @@ constexpr int kOffK = kOffQ + kTile;
 constexpr int kOffV = kOffK + kKStages * kTile;
 constexpr int kOffBar = kOffV + kVStages * kTile;
 constexpr int kSmemBytes = 1024 + kOffBar + 256;  // 1 KiB of alignment slack
+static_assert(kSmemBytes <= 227 * 1024, "shared memory");
 constexpr uint32_t kTmemCols = 512;
 // TMEM columns: S buffers at 0 and 128, O at 256, two P buffers (bf16 pairs
 // packed in 32-bit columns, 64 columns each) at 384 and 448.
