@@ -248,7 +248,9 @@ ps_status_t ps_kv_unpack(const void *src, const long long *src_offsets, const in
  *   q_start      int32 [num_seqs + 1], q_start[0] = 0, non-decreasing,
  *                q_start[num_seqs] <= total_q_tokens (all three on the device)
  *   max_q_len    an upper bound on Q_s over the batch (sizes the grid; the
- *                query tiles past a sequence's Q_s do nothing)
+ *                query tiles past a sequence's Q_s do nothing; a chunk longer
+ *                than max_q_len has its rows past it left unwritten and raises
+ *                PS_DEVICE_LEN_CLAMPED)
  *   device_status  optional device word that receives PS_DEVICE_* flags
  * A sequence with Q_s > seq_lens[s], a negative Q_s, a length above
  * max_blocks_per_seq * block_size or rows outside [0, total_q_tokens) is

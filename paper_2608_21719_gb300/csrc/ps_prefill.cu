@@ -272,6 +272,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int Q = qs1 - qs0;
     const int L = __ldg(p.seq_lens + s);
     const int tok0 = qt * tpt;
+    // max_q_len below a chunk leaves that chunk's later rows uncovered.
+    if (qt == p.num_qtiles - 1 && j == 0 && tid == 0 && Q > p.num_qtiles * tpt && p.status)
+        atomicOr(p.status, (unsigned)PS_DEVICE_LEN_CLAMPED);
     if (tok0 >= Q) return;
     const long long cap = (long long)p.max_blocks_per_seq * p.block_size;
     if (Q < 0 || L < Q || (long long)L > cap || qs0 < 0 || qs1 > p.total_q) {

@@ -225,3 +225,20 @@ def test_long_prompt_chunk_sampled_rows(psd):
     err = np.abs(got - ref)
     assert err.max() <= MAX_ABS, err.max()
     assert err.mean() <= MEAN_ABS, err.mean()
+
+
+def test_prefill_flags_a_chunk_longer_than_max_q_len(psd):
+    wl = inputs.make_prefill_workload("p1", device="cpu", new=[100, 20], prior=[30, 5], num_q_heads=8,
+                                      num_kv_heads=2, seed=12).to("cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    out = torch.full_like(wl.q, 5.0)
+    psd.prefill_attention(wl.q, wl.k_cache, wl.v_cache, wl.block_table, wl.seq_lens, wl.q_start, 40, out=out,
+                          scale=wl.scale, device_status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) & psd.PS_DEVICE_LEN_CLAMPED
+    ref = _oracle(wl)
+    # Rows inside the grid are right; the first sequence's rows past the
+    # grid (tiles of 32 tokens: rows 64..99) are untouched.
+    _compare(out[:64], ref[:64], "rows inside the grid")
+    _compare(out[100:], ref[100:], "second sequence")
+    assert torch.all(out[64:100] == 5.0)
