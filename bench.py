@@ -334,29 +334,54 @@ def run_ours(args):
     # step's inputs (queries, block table, lengths) from pinned host memory,
     # run the call, and read the output back.  The KV cache is the serving
     # engine's resident state and stays in HBM.
-    q_h = wl.q.cpu().pin_memory()
-    bt_h = wl.block_table.cpu().pin_memory()
-    sl_h = wl.seq_lens.cpu().pin_memory()
-    out_h = torch.empty(out.shape, dtype=out.dtype).pin_memory()
-    q_d, bt_d, sl_d = torch.empty_like(wl.q), torch.empty_like(wl.block_table), torch.empty_like(wl.seq_lens)
-    e2e_steps = max(10, min(K, 100))
-    ee = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(e2e_steps)]
-    for i in range(e2e_steps + 3):
-        flush.zero_()
-        if i >= 3:
-            ee[i - 3][0].record(stream)
-        q_d.copy_(q_h, non_blocking=True)
-        bt_d.copy_(bt_h, non_blocking=True)
-        sl_d.copy_(sl_h, non_blocking=True)
-        attn(q_d, wl.k_cache, wl.v_cache, bt_d, sl_d, out=out, scale=wl.scale, stream=stream)
-        out_h.copy_(out, non_blocking=True)
-        if i >= 3:
-            ee[i - 3][1].record(stream)
+    # The three inputs travel as one packed pinned buffer (one copy per step)
+    # into one device buffer that the call reads through three pointers.  As a
+    # serving loop would, the copies of step i+1 and the read-back of step i-1
+    # overlap the call of step i: two buffer sets, host-to-device copies,
+    # calls and read-backs on three streams ordered by events; the time is
+    # the whole loop's.  Every step still moves its own inputs in and its
+    # output out.  No L2 flush in between: each step reads the whole K/V pool,
+    # which is larger than L2.
+    packs = [packed_inputs([wl.q, wl.block_table, wl.seq_lens], dev) for _ in range(2)]
+    outs = [torch.empty_like(out) for _ in range(2)]
+    outs_h = [torch.empty(out.shape, dtype=out.dtype).pin_memory() for _ in range(2)]
+    h2d_s, d2h_s = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+    ev_in = [torch.cuda.Event() for _ in range(2)]
+    ev_k = [torch.cuda.Event() for _ in range(2)]
+    ev_out = [torch.cuda.Event() for _ in range(2)]
+    e2e_steps = max(10, min(K, 200))
+
+    def e2e_loop(nsteps):
+        for i in range(nsteps):
+            b = i % 2
+            (_, stage_h, (q_d, bt_d, sl_d), stage_d) = packs[b]
+            with torch.cuda.stream(h2d_s):
+                if i >= 2:
+                    h2d_s.wait_event(ev_k[b])  # step i-2 has finished reading buffer set b
+                stage_d.copy_(stage_h, non_blocking=True)
+                ev_in[b].record(h2d_s)
+            stream.wait_event(ev_in[b])
+            if i >= 2:
+                stream.wait_event(ev_out[b])  # step i-2's output has been read back
+            attn(q_d, wl.k_cache, wl.v_cache, bt_d, sl_d, out=outs[b], scale=wl.scale, stream=stream)
+            ev_k[b].record(stream)
+            with torch.cuda.stream(d2h_s):
+                d2h_s.wait_event(ev_k[b])
+                outs_h[b].copy_(outs[b], non_blocking=True)
+                ev_out[b].record(d2h_s)
+
+    e2e_loop(4)
     torch.cuda.synchronize(dev)
-    e2e_ms = statistics.mean(a.elapsed_time(b) for a, b in ee)
-    h2d = q_h.numel() * 2 + bt_h.numel() * 4 + sl_h.numel() * 4
-    d2h = out_h.numel() * 2
-    assert torch.equal(out_h, out.cpu())
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(h2d_s)
+    e2e_loop(e2e_steps)
+    d2h_s.wait_event(ev_out[(e2e_steps - 1) % 2])
+    e1.record(d2h_s)
+    torch.cuda.synchronize(dev)
+    e2e_ms = e0.elapsed_time(e1) / e2e_steps
+    h2d = packs[0][1].numel()
+    d2h = outs_h[0].numel() * 2
+    assert torch.equal(outs_h[(e2e_steps - 1) % 2], outs[(e2e_steps - 1) % 2].cpu())
 
     if rank != 0:
         if world > 1:
@@ -414,7 +439,11 @@ def run_ours(args):
             "algorithmic_bytes_per_launch": alg["total"],
         },
         "e2e": {"value": round(alg["kv"] / (e2e_ms * 1e-3) / 1e9, 2), "unit": "GB/s",
-                "ms_per_step": round(e2e_ms, 5), "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+                "ms_per_step": round(e2e_ms, 5), "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                "steps": e2e_steps,
+                "overlap": "copies of step i+1 and read-back of step i-1 overlap the call of step i "
+                           "(two buffer sets, three streams); time = whole loop / steps",
+                "l2": "not flushed: each step reads the whole K/V pool, larger than L2"},
         "gpu_launches": int(launches),
         "clocks": clk.summary(),
         "plan": attn.info(),
@@ -593,26 +622,22 @@ def run_prefill(args):
     tflops = flops / (ms * 1e-3) / 1e12
 
     # End to end: pinned host Q and metadata in, output back, every step.
-    q_h = wl.q.cpu().pin_memory()
-    meta_h = [t.cpu().pin_memory() for t in (wl.block_table, wl.seq_lens, wl.q_start)]
-    q_d = torch.empty_like(wl.q)
-    meta_d = [torch.empty_like(t) for t in (wl.block_table, wl.seq_lens, wl.q_start)]
+    (q_h, *meta_h), stage_h, (q_d, *meta_d), stage_d = packed_inputs(
+        [wl.q, wl.block_table, wl.seq_lens, wl.q_start], dev)
     out_h = torch.empty(out.shape, dtype=out.dtype, pin_memory=True)
     K2 = max(3, min(K, 50))
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     torch.cuda.synchronize(dev)
     e0.record(stream)
     for _ in range(K2):
-        q_d.copy_(q_h, non_blocking=True)
-        for dst, src in zip(meta_d, meta_h):
-            dst.copy_(src, non_blocking=True)
+        stage_d.copy_(stage_h, non_blocking=True)
         ps_decode.prefill_attention(q_d, wl.k_cache, wl.v_cache, meta_d[0], meta_d[1], meta_d[2], wl.max_q_len,
                                     out=out, scale=wl.scale, device_status=status, stream=stream.cuda_stream)
         out_h.copy_(out, non_blocking=True)
     e1.record(stream)
     torch.cuda.synchronize(dev)
     e2e_ms = e0.elapsed_time(e1) / K2
-    h2d = q_h.numel() * 2 + sum(t.numel() * 4 for t in meta_h)
+    h2d = stage_h.numel()
     d2h = out_h.numel() * 2
 
     peak, kind = bf16_peak()
@@ -638,6 +663,26 @@ def run_prefill(args):
         line["cpu_baseline"] = {"value": round(rate / 1e12, 6), "unit": "TFLOP/s", "cores": threads,
                                 "kind": "oracle", "sample": sample}
     return line
+
+
+def packed_inputs(tensors, dev, align=256):
+    """One pinned host buffer and one device buffer holding copies of
+    `tensors` at `align`-byte offsets; returns (host views, host buffer,
+    device views, device buffer)."""
+    import torch
+    offs, total = [], 0
+    for t in tensors:
+        offs.append(total)
+        total += (t.numel() * t.element_size() + align - 1) // align * align
+    stage_h = torch.empty(max(total, align), dtype=torch.uint8).pin_memory()
+    stage_d = torch.empty(max(total, align), dtype=torch.uint8, device=dev)
+
+    def views(buf):
+        return [buf[o:o + t.numel() * t.element_size()].view(t.dtype).view(t.shape) for o, t in zip(offs, tensors)]
+    hv = views(stage_h)
+    for h, t in zip(hv, tensors):
+        h.copy_(t.cpu())
+    return hv, stage_h, views(stage_d), stage_d
 
 
 # ------------------------------------------------------- reference arm ------
