@@ -35,6 +35,8 @@
 // the worker's outstanding copies with the same bound and returns.
 #include <cuda_bf16.h>
 
+#include <atomic>
+
 #include "ps_internal.h"
 
 namespace ps {
@@ -698,18 +700,29 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
 
 cudaError_t launch_decode(const DecodeParams &p, const CUtensorMap &tmK, const CUtensorMap &tmV, int grid_ctas,
                           size_t smem_bytes, cudaStream_t stream) {
-    // Raise the kernel's dynamic shared-memory limit (per device) whenever a
-    // launch needs more than any earlier one did.
-    static size_t attr_bytes[64] = {};
+    // Allow the kernel the largest dynamic shared memory the device offers
+    // (its opt-in limit less the kernel's static shared memory), once per
+    // device.  Every caller sets the same value, so concurrent first launches
+    // on one device cannot leave a smaller limit behind.
+    static std::atomic<int> attr_limit[64];
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-    if (smem_bytes > attr_bytes[dev]) {
-        e = cudaFuncSetAttribute(ps_decode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_bytes);
-        if (e != cudaSuccess) return e;
-        attr_bytes[dev] = smem_bytes;
+    int limit = attr_limit[dev].load(std::memory_order_acquire);
+    if (limit == 0) {
+        int optin = 0;
+        cudaFuncAttributes fa;
+        if ((e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev)) != cudaSuccess ||
+            (e = cudaFuncGetAttributes(&fa, ps_decode_kernel)) != cudaSuccess)
+            return e;
+        limit = optin - (int)fa.sharedSizeBytes;
+        if ((e = cudaFuncSetAttribute(ps_decode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, limit)) !=
+            cudaSuccess)
+            return e;
+        attr_limit[dev].store(limit, std::memory_order_release);
     }
+    if (smem_bytes > (size_t)limit) return cudaErrorInvalidValue;
     ps_decode_kernel<<<grid_ctas, kWorkersPerCta * 32, smem_bytes, stream>>>(p, tmK, tmV);
     return cudaGetLastError();
 }

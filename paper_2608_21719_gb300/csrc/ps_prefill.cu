@@ -616,12 +616,12 @@ extern "C" ps_status_t ps_prefill_attention(const void *q, const void *k_cache, 
         !encode3d(&tmK, k_cache, (cuuint64_t)block_size, (cuuint64_t)(num_blocks * num_kv_heads), kChunk, 1) ||
         !encode3d(&tmV, v_cache, (cuuint64_t)block_size, (cuuint64_t)(num_blocks * num_kv_heads), kChunk, 1))
         return PS_ERR_CUDA;
-    static std::once_flag attr_once;
-    static cudaError_t attr_err = cudaSuccess;
-    std::call_once(attr_once, [] {
-        attr_err = cudaFuncSetAttribute(ps_prefill_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
-    });
-    if (attr_err != cudaSuccess) return PS_ERR_CUDA;
+    // The shared-memory limit is a per-device function attribute: set it for
+    // the current device on every call (cheap), so that a process driving
+    // several GPUs works on each of them.
+    if (cudaFuncSetAttribute(ps_prefill_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) !=
+        cudaSuccess)
+        return PS_ERR_CUDA;
 
     PrefillParams pp;
     pp.block_table = block_table;
