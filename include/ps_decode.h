@@ -161,7 +161,11 @@ ps_status_t ps_decode_attention(const void *q, const void *k_cache, const void *
                                 int num_seqs, int num_q_heads, int num_kv_heads, int head_dim,
                                 int block_size, float scale, void *stream);
 
-/* The same computation with an explicit plan (no stream binding needed). */
+/* The same computation with an explicit plan (no stream binding needed).
+ * CUDA graphs: a call can be captured into a graph on `stream` once the plan
+ * has made one call outside capture with the same k_cache / v_cache (that
+ * call encodes the TMA descriptors on the host and clears the workspace's
+ * status word); replays then read whatever the captured pointers hold. */
 ps_status_t ps_decode_attention_planned(const ps_decode_plan_t *plan, const void *q,
                                         const void *k_cache, const void *v_cache,
                                         const int *block_table, const int *seq_lens, void *out,

@@ -137,6 +137,33 @@ def test_one_long_sequence_split_over_every_worker(psd):
     _compare(out, _oracle(wl), "L=131072")
 
 
+def test_planned_call_replays_in_a_cuda_graph(psd):
+    """A serving loop captures the decode step in a CUDA graph: after one
+    call outside capture (which encodes the tensor maps and clears the
+    workspace status), a captured planned call replays bit-identically."""
+    wl = _custom(32, 8, 16, [300, 1000, 17, 2048, 1, 4096], seed=21)
+    attn = psd.DecodeAttention.for_workload(wl)
+    out = torch.empty_like(wl.q)
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        attn(wl.q, wl.k_cache, wl.v_cache, wl.block_table, wl.seq_lens, out=out, scale=wl.scale, stream=side)
+    torch.cuda.synchronize()
+    ref = out.clone()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=side):
+        attn(wl.q, wl.k_cache, wl.v_cache, wl.block_table, wl.seq_lens, out=out, scale=wl.scale, stream=side)
+    for _ in range(2):
+        out.zero_()
+        torch.cuda.synchronize()
+        graph.replay()
+        torch.cuda.synchronize()
+        assert torch.equal(out, ref)
+    assert attn.device_status() == 0
+    attn.close()
+    _compare(ref, _oracle(wl), "graph")
+
+
 def test_repeated_calls_reuse_the_workspace_state(psd):
     # Segment counters return to zero after every call; a later call must
     # not see an earlier call's state, and the split is bit-deterministic.
