@@ -134,6 +134,15 @@ __device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *tm,
         "l"(reinterpret_cast<uint64_t>(tm)), "r"(c0), "r"(c1), "r"(c2), "r"(bar)
         : "memory");
 }
+// The same with an L2 cache-policy hint (from createpolicy).
+__device__ __forceinline__ void tma_load_3d_hint(uint32_t dst, const CUtensorMap *tm, int c0, int c1, int c2,
+                                                 uint32_t bar, uint64_t policy) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
+        " [%0], [%1, {%2, %3, %4}], [%5], %6;" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(tm)), "r"(c0), "r"(c1), "r"(c2), "r"(bar), "l"(policy)
+        : "memory");
+}
 __device__ __forceinline__ void tc_fence_before() {
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
 }
@@ -351,6 +360,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         const CUtensorMap *tm = is_k ? &tmK : &tmV;
         const int *bt_row = p.block_table + (size_t)s * p.max_blocks_per_seq;
         const int half = (lane >> 3) & 1, c = lane & 7;  // lanes 0-15: 8 chunks x 2 halves
+        // Every K/V page is read by all query tiles of its (sequence, head):
+        // ask L2 to keep it (evict last).
+        uint64_t keep;
+        asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(keep));
         int issued = 0;
         for (int n = 0; n < ntiles; ++n) {
             const int st = n % stages, use = n / stages;
@@ -369,8 +382,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 int page = -1;  // out of range: TMA fills zeros
                 if (b >= 0 && (long long)b < p.num_blocks) page = b * p.num_kv_heads + j;
                 else if (p.status && is_k) atomicOr(p.status, (unsigned)PS_DEVICE_BAD_BLOCK);
-                tma_load_3d(ring + st * kTile + half * kHalf + c * (kChunk * 128), tm, half * 64,
-                            t0 - lb * p.block_size, page, full);
+                tma_load_3d_hint(ring + st * kTile + half * kHalf + c * (kChunk * 128), tm, half * 64,
+                                 t0 - lb * p.block_size, page, full, keep);
             }
             issued = n + 1;
         }
