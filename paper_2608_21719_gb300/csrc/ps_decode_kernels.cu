@@ -113,6 +113,14 @@ __device__ __forceinline__ void bulk_load(uint32_t dst, const void *src, uint32_
         : "memory");
 }
 
+// 16-byte global -> shared copy that bypasses L1 (cp.async, completed by
+// cp.async.wait_all in the issuing thread).
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
+
 __device__ __forceinline__ void prefetch_l2(const void *p) {
     asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
 }
@@ -217,21 +225,126 @@ struct Partition {
 };
 
 // Merge `count` cut pieces of segment (s, h) into bf16 output rows by the
-// log-sum-exp rule.  Piece i's workspace slot comes from slot_lane(i), called
-// only by the lane that owns piece i (i = lane + 32k, may diverge), or from
-// slot_all(i), called by all lanes together with the same i.  Pieces are read
-// through L2 (other SMs wrote them).  Lanes take one piece each for the
-// (m, l) pass; for the weighted sums every lane owns dims [4*lane, 4*lane+4)
-// of every head, so all loads of a piece are in flight together.
-template <typename SlotLane, typename SlotAll>
-__device__ void merge_pieces(const DecodeParams &p, int count, SlotLane slot_lane, SlotAll slot_all, int s, int h,
-                             int lane) {
+// log-sum-exp rule.  Piece i's workspace slot is slot_of(i), evaluated by the
+// lane that owns piece i (i = lane + 32k, may diverge).  Pieces are read
+// through L2 (other SMs wrote them).  For the weighted sums every lane owns
+// dims [4*lane, 4*lane+4) of every head.
+//
+// The merge that completes a segment is usually the last thing its warp
+// does, so its latency adds to the kernel's tail.  Two paths:
+//  * staged (`stage` != nullptr: kStageArea bytes of this warp's shared
+//    memory that nothing else uses during the call, and count <= 32): the
+//    (m, l) pairs of all pieces and the accumulators of a batch of pieces are
+//    copied in with cp.async, all in flight together, and every lane then
+//    computes the maxima, weights and sums of l itself from broadcast reads,
+//    so the chain has one L2 round trip per batch and no shuffles (which are
+//    slow here while the other warps of the SM still stream);
+//  * otherwise (the ring is still streaming, or more than 32 pieces): lanes
+//    take one piece each for (m, l), reduce by shuffles, and read the
+//    accumulators one piece after another.
+constexpr int kStageArea = kWorkerBytes;
+constexpr int kStageMlBytes = 32 * (int)kSlotMl * 4;  // (m, l) of up to 32 pieces
+
+template <typename SlotOf>
+__device__ void merge_pieces_staged(const DecodeParams &p, int count, SlotOf slot_of, int s, int h, int lane,
+                                    uint8_t *stage) {
+    const int g = p.group;
+    const int per = min(32, (kStageArea - kStageMlBytes) / (g * kHeadDim * 4));  // pieces per acc batch
+    const uint32_t ml_base = smem_addr(stage);
+    const uint32_t acc_base = ml_base + kStageMlBytes + 16u * lane;
+    const uint8_t *ml_st = stage;
+    const uint8_t *acc_st = stage + kStageMlBytes + 16 * lane;
+    const int my_slot = lane < count ? (int)slot_of(lane) : 0;
+    if (lane < count) {
+        const float *src = p.ws_ml + (size_t)my_slot * kSlotMl;
+#pragma unroll
+        for (int c = 0; c < (int)kSlotMl / 4; ++c) cp_async16(ml_base + (uint32_t)(lane * kSlotMl + 4 * c) * 4, src + 4 * c);
+    }
+    auto issue_batch = [&](int first, int nb) {
+        for (int i = 0; i < nb; ++i) {
+            const float *src = p.ws_acc + (size_t)__shfl_sync(kFull, my_slot, first + i) * kSlotFloats + 4 * lane;
+            for (int n = 0; n < g; ++n)
+                cp_async16(acc_base + (uint32_t)(i * g + n) * (kHeadDim * 4), src + n * kHeadDim);
+        }
+    };
+    issue_batch(0, min(per, count));
+    cp_async_wait_all();
+    __syncwarp();  // (m, l) rows were copied by other lanes
+
+    float M[kMaxGroup];
+#pragma unroll
+    for (int n = 0; n < kMaxGroup; ++n) M[n] = -INFINITY;
+    for (int i = 0; i < count; ++i) {
+        const float4 *ml = reinterpret_cast<const float4 *>(ml_st + i * kSlotMl * 4);
+#pragma unroll
+        for (int q4 = 0; q4 < kMaxGroup / 2; ++q4) {
+            if (2 * q4 < g) {
+                const float4 v = ml[q4];
+                M[2 * q4] = fmaxf(M[2 * q4], v.x);
+                M[2 * q4 + 1] = fmaxf(M[2 * q4 + 1], v.z);
+            }
+        }
+    }
+    float4 acc[kMaxGroup];
+    float lsum[kMaxGroup];
+#pragma unroll
+    for (int n = 0; n < kMaxGroup; ++n) {
+        acc[n] = make_float4(0.f, 0.f, 0.f, 0.f);
+        lsum[n] = 0.f;
+    }
+    for (int jb = 0; jb < count; jb += per) {
+        const int nb = min(per, count - jb);
+        if (jb > 0) {
+            __syncwarp();
+            issue_batch(jb, nb);
+            cp_async_wait_all();
+        }
+        for (int i = 0; i < nb; ++i) {
+            const float4 *ml = reinterpret_cast<const float4 *>(ml_st + (jb + i) * kSlotMl * 4);
+            const uint8_t *src = acc_st + (size_t)i * g * (kHeadDim * 4);
+#pragma unroll
+            for (int q4 = 0; q4 < kMaxGroup / 2; ++q4) {
+                if (2 * q4 >= g) continue;
+                const float4 v = ml[q4];
+#pragma unroll
+                for (int k = 0; k < 2; ++k) {
+                    const int n = 2 * q4 + k;
+                    if (n < g) {
+                        const float en = ex2((k ? v.z : v.x) - M[n]);
+                        lsum[n] += en * (k ? v.w : v.y);
+                        const float4 a = *reinterpret_cast<const float4 *>(src + n * (kHeadDim * 4));
+                        acc[n].x += en * a.x; acc[n].y += en * a.y;
+                        acc[n].z += en * a.z; acc[n].w += en * a.w;
+                    }
+                }
+            }
+        }
+    }
+    uint16_t *o = p.out + ((size_t)s * p.num_q_heads + (size_t)h * g) * kHeadDim + 4 * lane;
+#pragma unroll
+    for (int n = 0; n < kMaxGroup; ++n) {
+        if (n < g) {
+            const float inv = 1.f / lsum[n];
+            const uint32_t lo = (uint32_t)f2bf(acc[n].x * inv) | ((uint32_t)f2bf(acc[n].y * inv) << 16);
+            const uint32_t hi = (uint32_t)f2bf(acc[n].z * inv) | ((uint32_t)f2bf(acc[n].w * inv) << 16);
+            *reinterpret_cast<uint2 *>(o + n * kHeadDim) = make_uint2(lo, hi);
+        }
+    }
+}
+
+template <typename SlotOf>
+__device__ void merge_pieces(const DecodeParams &p, int count, SlotOf slot_of, int s, int h, int lane,
+                             uint8_t *stage) {
+    if (stage != nullptr && count <= 32) {
+        merge_pieces_staged(p, count, slot_of, s, h, lane, stage);
+        return;
+    }
     const int g = p.group;
     float M[kMaxGroup];
 #pragma unroll
     for (int n = 0; n < kMaxGroup; ++n) M[n] = -INFINITY;
     for (int i = lane; i < count; i += 32) {
-        const float4 *ml = reinterpret_cast<const float4 *>(p.ws_ml + slot_lane(i) * kSlotMl);
+        const float4 *ml = reinterpret_cast<const float4 *>(p.ws_ml + slot_of(i) * kSlotMl);
 #pragma unroll
         for (int q4 = 0; q4 < kMaxGroup / 2; ++q4) {
             const float4 v = __ldcg(ml + q4);
@@ -241,8 +354,9 @@ __device__ void merge_pieces(const DecodeParams &p, int count, SlotLane slot_lan
     }
 #pragma unroll
     for (int n = 0; n < kMaxGroup; ++n)
+        if (n < g)
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) M[n] = fmaxf(M[n], __shfl_xor_sync(kFull, M[n], o));
+            for (int o = 16; o > 0; o >>= 1) M[n] = fmaxf(M[n], __shfl_xor_sync(kFull, M[n], o));
     float4 acc[kMaxGroup];
     float lsum[kMaxGroup];
 #pragma unroll
@@ -251,9 +365,10 @@ __device__ void merge_pieces(const DecodeParams &p, int count, SlotLane slot_lan
         lsum[n] = 0.f;
     }
     for (int ib = 0; ib < count; ib += 32) {
+        const int my_slot = ib + lane < count ? (int)slot_of(ib + lane) : 0;
         float e[kMaxGroup];
         if (ib + lane < count) {
-            const float4 *ml = reinterpret_cast<const float4 *>(p.ws_ml + slot_lane(ib + lane) * kSlotMl);
+            const float4 *ml = reinterpret_cast<const float4 *>(p.ws_ml + (size_t)my_slot * kSlotMl);
 #pragma unroll
             for (int q4 = 0; q4 < kMaxGroup / 2; ++q4) {
                 const float4 v = __ldcg(ml + q4);
@@ -268,33 +383,31 @@ __device__ void merge_pieces(const DecodeParams &p, int count, SlotLane slot_lan
         }
         const int cnt = min(32, count - ib);
         for (int i = 0; i < cnt; ++i) {
-            const float *src = p.ws_acc + slot_all(ib + i) * kSlotFloats + 4 * lane;
+            const float *src = p.ws_acc + (size_t)__shfl_sync(kFull, my_slot, i) * kSlotFloats + 4 * lane;
             float4 v[kMaxGroup];
 #pragma unroll
             for (int n = 0; n < kMaxGroup; ++n)
                 if (n < g) v[n] = __ldcg(reinterpret_cast<const float4 *>(src + n * kHeadDim));
 #pragma unroll
             for (int n = 0; n < kMaxGroup; ++n) {
-                const float en = __shfl_sync(kFull, e[n], i);
                 if (n < g) {
+                    const float en = __shfl_sync(kFull, e[n], i);
                     acc[n].x += en * v[n].x; acc[n].y += en * v[n].y;
                     acc[n].z += en * v[n].z; acc[n].w += en * v[n].w;
                 }
             }
         }
     }
-#pragma unroll
-    for (int n = 0; n < kMaxGroup; ++n)
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) lsum[n] += __shfl_xor_sync(kFull, lsum[n], o);
     uint16_t *o = p.out + ((size_t)s * p.num_q_heads + (size_t)h * g) * kHeadDim + 4 * lane;
 #pragma unroll
     for (int n = 0; n < kMaxGroup; ++n) {
         if (n < g) {
+#pragma unroll
+            for (int sh = 16; sh > 0; sh >>= 1) lsum[n] += __shfl_xor_sync(kFull, lsum[n], sh);
             const float inv = 1.f / lsum[n];
-            uint16_t *on = o + n * kHeadDim;
-            on[0] = f2bf(acc[n].x * inv); on[1] = f2bf(acc[n].y * inv);
-            on[2] = f2bf(acc[n].z * inv); on[3] = f2bf(acc[n].w * inv);
+            const uint32_t lo = (uint32_t)f2bf(acc[n].x * inv) | ((uint32_t)f2bf(acc[n].y * inv) << 16);
+            const uint32_t hi = (uint32_t)f2bf(acc[n].z * inv) | ((uint32_t)f2bf(acc[n].w * inv) << 16);
+            *reinterpret_cast<uint2 *>(o + n * kHeadDim) = make_uint2(lo, hi);
         }
     }
 }
@@ -495,7 +608,7 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
 
     // Finish the consume side's current piece: write its output, or leave its
     // partial state and count its tiles, merging the segment if it was last.
-    auto finalize = [&]() {
+    auto finalize = [&](bool ring_idle) {
         float L0 = l0, L1 = l1;
 #pragma unroll
         for (int o = 4; o < 32; o <<= 1) {
@@ -557,7 +670,7 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
             const int r = r0 + i;
             return 2 * (size_t)r + (part.range_begin(r) < a ? 1 : 0);
         };
-        merge_pieces(p, r1 - r0 + 1, slot_of, slot_of, s, h, lane);
+        merge_pieces(p, r1 - r0 + 1, slot_of, s, h, lane, ring_idle ? wbase : nullptr);
         if (lane == 0) *cnt = 0;
     };
 
@@ -578,7 +691,7 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
         const int4 meta = wmeta[slot];
         const int st = meta.x, pord = meta.y;
         if (pord != cur_piece) {
-            if (cur_piece >= 0) finalize();
+            if (cur_piece >= 0) finalize(false);
             cur_piece = pord;
             cpi = wpieces[pord & 3];
             const uint32_t qs = smem_addr(qslots + (pord % kQSlots) * kQSlotBytes);
@@ -693,7 +806,8 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
         ++consumed;
         refill(consumed);
     }
-    if (cur_piece >= 0) finalize();
+    // Every copy into the ring has landed: it can stage the final merge.
+    if (cur_piece >= 0) finalize(true);
 }
 
 }  // namespace
