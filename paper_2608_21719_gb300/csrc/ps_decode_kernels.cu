@@ -240,9 +240,19 @@ struct Partition {
 //    so the chain has one L2 round trip per batch and no shuffles (which are
 //    slow here while the other warps of the SM still stream);
 //  * otherwise (the ring is still streaming, or more than 32 pieces): lanes
-//    take one piece each for (m, l), reduce by shuffles, and read the
-//    accumulators one piece after another.
+//    take one piece each for (m, l), reduce the maxima by shuffles, and read
+//    the accumulators one piece after another.
+// Both paths add the pieces' terms in piece order with the same operations,
+// so the output bits do not depend on which warp merged, or where.
 constexpr int kStageArea = kWorkerBytes;
+
+// One piece's contribution to the merged sums (explicit fma).
+__device__ __forceinline__ void accumulate_piece(float4 &acc, float &lsum, float e, float l, const float4 &a) {
+    lsum = fmaf(e, l, lsum);
+    acc.x = fmaf(e, a.x, acc.x); acc.y = fmaf(e, a.y, acc.y);
+    acc.z = fmaf(e, a.z, acc.z); acc.w = fmaf(e, a.w, acc.w);
+}
+
 constexpr int kStageMlBytes = 32 * (int)kSlotMl * 4;  // (m, l) of up to 32 pieces
 
 template <typename SlotOf>
@@ -311,10 +321,8 @@ __device__ void merge_pieces_staged(const DecodeParams &p, int count, SlotOf slo
                     const int n = 2 * q4 + k;
                     if (n < g) {
                         const float en = ex2((k ? v.z : v.x) - M[n]);
-                        lsum[n] += en * (k ? v.w : v.y);
                         const float4 a = *reinterpret_cast<const float4 *>(src + n * (kHeadDim * 4));
-                        acc[n].x += en * a.x; acc[n].y += en * a.y;
-                        acc[n].z += en * a.z; acc[n].w += en * a.w;
+                        accumulate_piece(acc[n], lsum[n], en, k ? v.w : v.y, a);
                     }
                 }
             }
@@ -333,12 +341,7 @@ __device__ void merge_pieces_staged(const DecodeParams &p, int count, SlotOf slo
 }
 
 template <typename SlotOf>
-__device__ void merge_pieces(const DecodeParams &p, int count, SlotOf slot_of, int s, int h, int lane,
-                             uint8_t *stage) {
-    if (stage != nullptr && count <= 32) {
-        merge_pieces_staged(p, count, slot_of, s, h, lane, stage);
-        return;
-    }
+__device__ void merge_pieces_direct(const DecodeParams &p, int count, SlotOf slot_of, int s, int h, int lane) {
     const int g = p.group;
     float M[kMaxGroup];
 #pragma unroll
@@ -366,20 +369,22 @@ __device__ void merge_pieces(const DecodeParams &p, int count, SlotOf slot_of, i
     }
     for (int ib = 0; ib < count; ib += 32) {
         const int my_slot = ib + lane < count ? (int)slot_of(ib + lane) : 0;
-        float e[kMaxGroup];
+        float e[kMaxGroup], l[kMaxGroup];  // weight and l of piece ib + lane
+#pragma unroll
+        for (int n = 0; n < kMaxGroup; ++n) e[n] = l[n] = 0.f;
         if (ib + lane < count) {
             const float4 *ml = reinterpret_cast<const float4 *>(p.ws_ml + (size_t)my_slot * kSlotMl);
 #pragma unroll
             for (int q4 = 0; q4 < kMaxGroup / 2; ++q4) {
+                if (2 * q4 >= g) continue;
                 const float4 v = __ldcg(ml + q4);
-                e[2 * q4] = 2 * q4 < g ? ex2(v.x - M[2 * q4]) : 0.f;
-                e[2 * q4 + 1] = 2 * q4 + 1 < g ? ex2(v.z - M[2 * q4 + 1]) : 0.f;
-                lsum[2 * q4] += e[2 * q4] * v.y;
-                lsum[2 * q4 + 1] += e[2 * q4 + 1] * v.w;
+                e[2 * q4] = ex2(v.x - M[2 * q4]);
+                l[2 * q4] = v.y;
+                if (2 * q4 + 1 < g) {
+                    e[2 * q4 + 1] = ex2(v.z - M[2 * q4 + 1]);
+                    l[2 * q4 + 1] = v.w;
+                }
             }
-        } else {
-#pragma unroll
-            for (int n = 0; n < kMaxGroup; ++n) e[n] = 0.f;
         }
         const int cnt = min(32, count - ib);
         for (int i = 0; i < cnt; ++i) {
@@ -389,27 +394,28 @@ __device__ void merge_pieces(const DecodeParams &p, int count, SlotOf slot_of, i
             for (int n = 0; n < kMaxGroup; ++n)
                 if (n < g) v[n] = __ldcg(reinterpret_cast<const float4 *>(src + n * kHeadDim));
 #pragma unroll
-            for (int n = 0; n < kMaxGroup; ++n) {
-                if (n < g) {
-                    const float en = __shfl_sync(kFull, e[n], i);
-                    acc[n].x += en * v[n].x; acc[n].y += en * v[n].y;
-                    acc[n].z += en * v[n].z; acc[n].w += en * v[n].w;
-                }
-            }
+            for (int n = 0; n < kMaxGroup; ++n)
+                if (n < g)
+                    accumulate_piece(acc[n], lsum[n], __shfl_sync(kFull, e[n], i), __shfl_sync(kFull, l[n], i), v[n]);
         }
     }
     uint16_t *o = p.out + ((size_t)s * p.num_q_heads + (size_t)h * g) * kHeadDim + 4 * lane;
 #pragma unroll
     for (int n = 0; n < kMaxGroup; ++n) {
         if (n < g) {
-#pragma unroll
-            for (int sh = 16; sh > 0; sh >>= 1) lsum[n] += __shfl_xor_sync(kFull, lsum[n], sh);
             const float inv = 1.f / lsum[n];
             const uint32_t lo = (uint32_t)f2bf(acc[n].x * inv) | ((uint32_t)f2bf(acc[n].y * inv) << 16);
             const uint32_t hi = (uint32_t)f2bf(acc[n].z * inv) | ((uint32_t)f2bf(acc[n].w * inv) << 16);
             *reinterpret_cast<uint2 *>(o + n * kHeadDim) = make_uint2(lo, hi);
         }
     }
+}
+
+template <typename SlotOf>
+__device__ __forceinline__ void merge_pieces(const DecodeParams &p, int count, SlotOf slot_of, int s, int h, int lane,
+                                             uint8_t *stage) {
+    if (stage != nullptr && count <= 32) merge_pieces_staged(p, count, slot_of, s, h, lane, stage);
+    else merge_pieces_direct(p, count, slot_of, s, h, lane);
 }
 
 // --------------------------------------------------------------- kernel ----
