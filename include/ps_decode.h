@@ -112,9 +112,10 @@ ps_status_t ps_decode_plan_create(int num_seqs, int num_q_heads, int num_kv_head
 /*
  * As ps_decode_plan_create(), with explicit knobs (0 = default for each):
  *   num_sms                SM count to size the grid for (0: query the device;
- *                          a positive value needs no GPU, e.g. for host tests)
- *   max_workers            upper bound on the number of equal contiguous
- *                          ranges the batch's KV stream is split into
+ *                          a positive value needs no GPU, e.g. for host tests;
+ *                          at most 4096, else PS_ERR_UNSUPPORTED)
+ *   max_workers            upper bound on the number of contiguous ranges of
+ *                          equal cost the batch's KV stream is split into
  *                          (1 = one warp does everything, no split)
  *   min_stages_per_worker  smallest range, in 16-token tiles
  *                          (1 = split as finely as the workers allow)

@@ -54,10 +54,11 @@ ps_status_t check_shape(int num_seqs, int num_q_heads, int num_kv_heads, int hea
     if (num_q_heads / num_kv_heads > kMaxGroup) return PS_ERR_UNSUPPORTED;
     if (block_size % kTileTokens != 0 || block_size > 256) return PS_ERR_UNSUPPORTED;
     if (num_seqs > kMaxSeqs || partial_smem_bytes(num_seqs) > kMaxSmemPerCta) return PS_ERR_UNSUPPORTED;
-    // Tile counts and TMA row coordinates are 32-bit.
+    // Tile counts, the split's cost units and TMA row coordinates are 32-bit.
     const long long len_cap = (long long)max_blocks_per_seq * block_size;
     const long long tiles = (long long)num_seqs * ((len_cap + kTileTokens - 1) / kTileTokens) * num_kv_heads;
-    if (len_cap > INT32_MAX || tiles > INT32_MAX) return PS_ERR_UNSUPPORTED;
+    const long long units = tiles + (long long)kSegmentCost * num_kv_heads * num_seqs;
+    if (len_cap > INT32_MAX || units > INT32_MAX) return PS_ERR_UNSUPPORTED;
     if (num_blocks * num_kv_heads > INT32_MAX) return PS_ERR_UNSUPPORTED;
     return PS_OK;
 }
@@ -173,6 +174,7 @@ ps_status_t ps_decode_plan_create_ex(int num_seqs, int num_q_heads, int num_kv_h
     *plan = nullptr;
     *workspace_bytes = 0;
     if (num_sms < 0 || max_workers < 0 || min_stages_per_worker < 0) return PS_ERR_INVALID_ARG;
+    if (num_sms > kMaxGridCtas) return PS_ERR_UNSUPPORTED;
     ps_status_t e = check_shape(num_seqs, num_q_heads, num_kv_heads, head_dim, block_size, max_blocks_per_seq,
                                 num_blocks);
     if (e != PS_OK) return e;

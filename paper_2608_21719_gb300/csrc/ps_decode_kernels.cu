@@ -188,21 +188,6 @@ struct Cursor {
 
 __device__ __forceinline__ int tiles_of(int len) { return (len + kTileTokens - 1) / kTileTokens; }
 
-__device__ __forceinline__ Cursor locate(const int *sP, const int *sL, int S, int x) {
-    int lo = 0, hi = S - 1;
-    while (lo < hi) {
-        const int mid = (lo + hi + 1) >> 1;
-        if (sP[mid] <= x) lo = mid; else hi = mid - 1;
-    }
-    Cursor c;
-    c.s = lo;
-    c.ns = tiles_of(sL[lo]);
-    const int off = x - sP[lo];
-    c.h = off / c.ns;
-    c.st = off - c.h * c.ns;
-    return c;
-}
-
 __device__ __forceinline__ void advance(Cursor &c, const int *sL, int S, int Hkv) {
     if (++c.st < c.ns) return;
     c.st = 0;
@@ -214,14 +199,94 @@ __device__ __forceinline__ void advance(Cursor &c, const int *sL, int S, int Hkv
     c.ns = c.s < S ? tiles_of(sL[c.s]) : 0;
 }
 
-// Split of the tape into Ws equal contiguous static ranges; range r covers
-// tiles [floor(r N / Ws), floor((r+1) N / Ws)).
+// Split of the tape into Ws contiguous static ranges of equal cost.  A warp
+// loses time at each segment boundary inside its range (the cut piece's
+// partial state and counter update, the next segment's query and
+// block-table window), so a segment of ns tiles costs ns + c units, with
+// c = kSegmentCost, and ranges are equal in units.  When ranges average
+// fewer than 8c tiles (small, latency-bound batches) c is 0: the plain
+// equal split.  Unit positions have a closed form: sequence s starts at
+// U(s) = sP[s] + c * Hkv * s (an empty sequence costs c per head as well),
+// segment h of it at U(s) + h * (ns + c), and its tiles take the first ns
+// units.  Range r covers units [floor(r Utot / Ws), floor((r+1) Utot / Ws)).
+// All of it is 32-bit: the host bounds Utot below 2^31 and the grid's
+// workers below 2^15 (so r * (Utot mod Ws) < 2^30).
 struct Partition {
-    int N, Ws;
+    int N, Ws, S, Hkv, c, Utot, q0, r0;  // Utot = q0 * Ws + r0
+    float ws_rcp, ws_per_unit;
+    const int *sP, *sL;
 
-    __device__ int range_of(int x) const { return (int)((((long long)x + 1) * Ws - 1) / N); }
-    __device__ int range_begin(int r) const { return (int)((long long)r * N / Ws); }
-    __device__ int range_end(int r) const { return (int)((long long)(r + 1) * N / Ws); }
+    __device__ void init(int N_, int Ws_, int S_, int Hkv_, const int *sP_, const int *sL_) {
+        N = N_; Ws = Ws_; S = S_; Hkv = Hkv_; sP = sP_; sL = sL_;
+        c = (long long)N >= 8LL * kSegmentCost * Ws ? kSegmentCost : 0;
+        Utot = seq_unit(S);
+        q0 = Ws > 0 ? Utot / Ws : 0;
+        r0 = Utot - q0 * Ws;
+        ws_rcp = 1.f / (float)max(Ws, 1);
+        ws_per_unit = (float)Ws / (float)max(Utot, 1);
+    }
+    __device__ int seq_unit(int s) const { return sP[s] + c * Hkv * s; }
+    __device__ int segment_unit(int s, int h, int ns) const { return seq_unit(s) + h * (ns + c); }
+    // floor(r Utot / Ws) = r q0 + floor(r r0 / Ws); the last quotient is below
+    // Ws <= 2^15, so a float estimate is off by at most one and is corrected.
+    __device__ int unit_begin(int r) const {
+        const int x = r * r0;
+        int q = (int)((float)x * ws_rcp);
+        q += (q + 1) * Ws <= x ? 1 : 0;
+        q -= q * Ws > x ? 1 : 0;
+        return r * q0 + q;
+    }
+    // The range holding unit u: a float estimate, corrected exactly.
+    __device__ int range_of_unit(int u) const {
+        int r = min(Ws - 1, (int)((float)u * ws_per_unit));
+        while (r + 1 < Ws && unit_begin(r + 1) <= u) ++r;
+        while (r > 0 && unit_begin(r) > u) --r;
+        return r;
+    }
+    // Where unit u falls (one lane): sequence s, head h, offset o in the
+    // segment's ns + c units, and the number of tiles before u.
+    struct Pos {
+        int tile, s, h, o, ns;
+    };
+    __device__ Pos position(int u) const {
+        Pos q;
+        if (u >= Utot) {
+            q.tile = N; q.s = S; q.h = 0; q.o = 0; q.ns = 0;
+            return q;
+        }
+        int lo = 0, hi = S - 1;
+        while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (seq_unit(mid) <= u) lo = mid; else hi = mid - 1;
+        }
+        q.s = lo;
+        q.ns = tiles_of(sL[lo]);
+        const int off = u - seq_unit(lo);  // < Hkv * (ns + c)
+        const int d = q.ns + c;             // >= 1: the sequence holding u has units
+        int h = (int)((float)off * __frcp_rn((float)d));  // h < Hkv: off by at most one
+        h += (h + 1) * d <= off ? 1 : 0;
+        h -= h * d > off ? 1 : 0;
+        q.h = h;
+        q.o = off - h * d;
+        q.tile = sP[lo] + q.h * q.ns + min(q.o, q.ns);
+        return q;
+    }
+    // The ranges r0..r1 holding segment (s, h) (tiles a .. a+ns-1), and
+    // whether range r0 began at an earlier tile (then the segment's piece is
+    // r0's second piece).  The merging warp's own range w = [b, e) is
+    // usually r0 or r1, which needs no arithmetic.
+    __device__ void merge_bounds(int s, int h, int ns, int w, int b, int e, int &r0, int &r1, int &cut0) const {
+        const int a = sP[s] + h * ns;
+        const int ua = segment_unit(s, h, ns);
+        if (a >= b && a < e) {
+            r0 = w;
+            cut0 = b < a ? 1 : 0;
+        } else {
+            r0 = range_of_unit(ua);
+            cut0 = position(unit_begin(r0)).tile < a ? 1 : 0;
+        }
+        r1 = (a + ns - 1 >= b && a + ns - 1 < e) ? w : range_of_unit(ua + ns - 1);
+    }
 };
 
 // Merge `count` cut pieces of segment (s, h) into bf16 output rows by the
@@ -484,11 +549,11 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
 
     // 2. Partition of the tape (identical in every CTA).
     Partition part;
-    const int W = gridDim.x * kWorkersPerCta;
-    part.N = sP[S];
     {
-        const int cap = (part.N + p.min_stages - 1) / p.min_stages;
-        part.Ws = part.N > 0 ? max(1, min(min(W, p.max_workers), cap)) : 0;
+        const int N = sP[S];
+        const int W = gridDim.x * kWorkersPerCta;
+        const int cap = (N + p.min_stages - 1) / p.min_stages;
+        part.init(N, N > 0 ? max(1, min(min(W, p.max_workers), cap)) : 0, S, Hkv, sP, sL);
     }
     const int w = warp * gridDim.x + blockIdx.x;  // CTAs first: a small Ws still spreads over SMs
 
@@ -500,14 +565,33 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
     const int mbps = p.max_blocks_per_seq;
 
     // ---- issue side: TMA producer state (lane 0 issues, all lanes track) ----
-    bool issuing = w < part.Ws;
+    const bool issuing = w < part.Ws;
     int cur_rid = w, cur_b = 0, cur_e = 0, ip = 0;
     Cursor ic{0, 0, 0, 0};
     if (issuing) {
-        cur_b = part.range_begin(w);
-        cur_e = part.range_end(w);
+        // Lanes 0 and 1 find where the range starts and ends, at once.
+        const Partition::Pos q = part.position(part.unit_begin(w + (lane & 1)));
+        cur_b = __shfl_sync(kFull, q.tile, 0);
+        cur_e = __shfl_sync(kFull, q.tile, 1);
         ip = cur_b;
-        ic = locate(sP, sL, S, ip);
+        ic.s = __shfl_sync(kFull, q.s, 0);
+        ic.h = __shfl_sync(kFull, q.h, 0);
+        ic.st = __shfl_sync(kFull, q.o, 0);
+        ic.ns = __shfl_sync(kFull, q.ns, 0);
+        if (cur_b < cur_e && ic.st >= ic.ns) {
+            // The start is in boundary units: the range begins at the next
+            // segment (a range can also hold boundary units only).
+            ic.st = 0;
+            if (ic.ns > 0 && ic.h + 1 < Hkv) {
+                ++ic.h;
+            } else {
+                ic.h = 0;
+                do {
+                    ++ic.s;
+                } while (sL[ic.s] == 0);
+                ic.ns = tiles_of(sL[ic.s]);
+            }
+        }
     }
 
     int issued = 0, pieces_issued = 0;
@@ -670,12 +754,11 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
         if (done != ns) return;
         // This warp completed the segment: merge its pieces in tape order.
         __threadfence();
-        const int a = sP[s] + h * ns;
-        const int r0 = part.range_of(a), r1 = part.range_of(a + ns - 1);
-        auto slot_of = [&](int i) -> size_t {
-            const int r = r0 + i;
-            return 2 * (size_t)r + (part.range_begin(r) < a ? 1 : 0);
-        };
+        // Range r0 + i holds one piece of the segment: its first piece (slot
+        // 2r) unless the range began at an earlier tile.  Only r0 can.
+        int r0, r1, cut0;
+        part.merge_bounds(s, h, ns, cur_rid, cur_b, cur_e, r0, r1, cut0);
+        auto slot_of = [&](int i) -> size_t { return 2 * (size_t)(r0 + i) + (i == 0 ? cut0 : 0); };
         merge_pieces(p, r1 - r0 + 1, slot_of, s, h, lane, ring_idle ? wbase : nullptr);
         if (lane == 0) *cnt = 0;
     };

@@ -32,6 +32,15 @@ constexpr int kStages = PS_STAGES;
 #define PS_QSLOTS 2
 #endif
 constexpr int kQSlots = PS_QSLOTS;       // query tiles staged per warp
+// Weight of a segment boundary in the static split, in tiles: a warp loses
+// ~2-3 tiles' time at each one (measured); 4 was the best of 0-6 on the four
+// large workloads together (the response is not smooth: boundary placement
+// matters as well).
+#ifndef PS_SEGMENT_COST
+#define PS_SEGMENT_COST 4
+#endif
+constexpr int kSegmentCost = PS_SEGMENT_COST;
+constexpr int kMaxGridCtas = 4096;             // keeps the split's 32-bit arithmetic exact
 constexpr int kDefaultMinStages = 2;     // smallest share of a worker, in tiles (tuned on the 4-sequence workload)
 
 // Shared-memory geometry.  A 16-token x 128-dim bf16 tile is loaded as two

@@ -79,6 +79,9 @@ def test_max_seqs_plan_fits_shared_memory():
     (dict(num_seqs=4097), psd.PS_ERR_UNSUPPORTED),
     (dict(num_blocks=0), psd.PS_ERR_INVALID_ARG),
     (dict(num_sms=-1), psd.PS_ERR_INVALID_ARG),
+    (dict(num_sms=4097), psd.PS_ERR_UNSUPPORTED),  # the split's 32-bit arithmetic needs < 2^15 workers
+    # 4096 sequences x 8 heads x 65536 tiles: tile and cost-unit counts past 2^31
+    (dict(num_seqs=4096, num_kv_heads=8, num_q_heads=64, max_blocks_per_seq=65536), psd.PS_ERR_UNSUPPORTED),
 ])
 def test_plan_rejects_bad_shapes(kw, status):
     with pytest.raises(psd.PsError) as ei:

@@ -108,6 +108,22 @@ def test_forced_splits(psd, max_workers, min_stages):
     _compare(out, _oracle(wl), "split %s/%s" % (max_workers, min_stages))
 
 
+@pytest.mark.parametrize("max_workers,min_stages", [(0, 1), (40, 1), (57, 2)])
+def test_split_with_ranges_of_boundary_units_only(psd, max_workers, min_stages):
+    # Each segment costs its tiles plus a fixed number of boundary units in
+    # the static split; with many empty and one-tile sequences and ranges of
+    # one or two units, some ranges hold boundary units only (no tiles) and
+    # others start right at a segment.
+    lengths = [0, 1, 0, 0, 16, 17, 0, 3, 33, 0, 1, 48, 0, 0, 5, 250, 0, 1, 1, 1]
+    wl = _custom(16, 4, 16, lengths, seed=21, spare=9)
+    out, status, info = _gpu(psd, wl, max_workers=max_workers, min_stages_per_worker=min_stages)
+    assert status == 0
+    _compare(out, _oracle(wl), "boundary-only ranges %d/%d" % (max_workers, min_stages))
+    for s, L in enumerate(lengths):
+        if L == 0:
+            assert torch.all(out[s] == 0)
+
+
 def test_maximum_number_of_sequences(psd):
     """4096 sequences (the limit of the per-CTA length tables), ragged and
     partly empty, all compared with the oracle."""
