@@ -326,6 +326,27 @@ ps_status_t ps_decode_attention_noalloc(const void *q, const void *k_cache, cons
                                         int block_size, int max_blocks_per_seq, long long num_blocks,
                                         float scale, void *stream);
 
+/*
+ * Fault injection, for tests of the error paths (process-wide, one shot,
+ * value 0 clears; nothing here faults, traps or hangs the GPU):
+ *   PS_INJECT_LAUNCH_ERROR  the library's next kernel launch, from any entry
+ *                           point, is not made; the call returns PS_ERR_CUDA
+ *                           as if the launch had reported CUDA error `value`
+ *                           (1 .. 10000).
+ *   PS_INJECT_DECODE_STALL  the next decode-attention launch makes every
+ *                           streaming warp first wait, for `value` ns
+ *                           (1000 .. 1000000000), on an mbarrier that nothing
+ *                           arrives on.  The wait runs out as a real stall
+ *                           would: the kernel raises PS_DEVICE_TIMEOUT, lets
+ *                           the copies it has in flight land and exits
+ *                           without writing any output (which is then
+ *                           invalid).  Recovery is the documented one.
+ * Errors: PS_ERR_INVALID_ARG for an unknown kind or a value out of range.
+ */
+#define PS_INJECT_LAUNCH_ERROR 1
+#define PS_INJECT_DECODE_STALL 2
+ps_status_t ps_test_inject(int kind, long long value);
+
 /* Number of kernels this library has launched in this process through the
  * decode, fused-append, prefill and KV hand-off entry points (the
  * workspace-free entry point is not counted). */

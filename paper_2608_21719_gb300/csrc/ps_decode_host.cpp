@@ -165,6 +165,32 @@ ps_status_t run_planned(ps_decode_plan *p, const void *q, const void *k, const v
 
 void ps::note_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 
+namespace {
+std::atomic<int> g_inject_launch_error{0};
+std::atomic<long long> g_inject_stall_ns{0};
+}  // namespace
+
+cudaError_t ps::take_injected_launch_error() {
+    return static_cast<cudaError_t>(g_inject_launch_error.exchange(0, std::memory_order_acq_rel));
+}
+
+long long ps::take_injected_stall_ns() { return g_inject_stall_ns.exchange(0, std::memory_order_acq_rel); }
+
+ps_status_t ps_test_inject(int kind, long long value) {
+    switch (kind) {
+        case PS_INJECT_LAUNCH_ERROR:
+            if (value < 0 || value > 10000) return PS_ERR_INVALID_ARG;
+            g_inject_launch_error.store((int)value, std::memory_order_release);
+            return PS_OK;
+        case PS_INJECT_DECODE_STALL:
+            if (value != 0 && (value < 1000 || value > 1000000000)) return PS_ERR_INVALID_ARG;
+            g_inject_stall_ns.store(value, std::memory_order_release);
+            return PS_OK;
+        default:
+            return PS_ERR_INVALID_ARG;
+    }
+}
+
 extern "C" {
 
 ps_status_t ps_decode_plan_create_ex(int num_seqs, int num_q_heads, int num_kv_heads, int head_dim, int block_size,

@@ -87,13 +87,15 @@ __device__ __forceinline__ unsigned long long global_ns() {
     return t;
 }
 
-// Bounded wait for phase `parity` of an mbarrier; false after ~2 s.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+// Bounded wait for phase `parity` of an mbarrier; false after limit_ns
+// (~2 s by default).
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity,
+                                          unsigned long long limit_ns = kWaitLimitNs) {
     for (int i = 0; i < 256; ++i)
         if (mbar_try_wait(bar, parity)) return true;
     const unsigned long long t0 = global_ns();
     while (!mbar_try_wait(bar, parity))
-        if (global_ns() - t0 > kWaitLimitNs) return false;
+        if (global_ns() - t0 > limit_ns) return false;
     return true;
 }
 
@@ -496,6 +498,7 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
     int *sP = reinterpret_cast<int *>(pieces + kWorkersPerCta * 4);           // [S + 1] tile prefix (x Hkv)
     int *sL = sP + p.num_seqs + 1;                                            // [S] clamped lengths
     __shared__ int warp_sums[kWorkersPerCta];
+    __shared__ uint64_t stall_bar;  // nothing arrives on it: the injected stall (tests only)
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int S = p.num_seqs, Hkv = p.num_kv_heads, g = p.group, bs = p.block_size;
@@ -537,6 +540,7 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
         if (lo < hi && hi == S) sP[S] = run;
         if (lane == 0)
             for (int i = 0; i < kStages; ++i) mbar_init(smem_addr(&bars[warp * kStages + i]), 1);
+        if (tid == 0) mbar_init(smem_addr(&stall_bar), 1);
         fence_mbar_init();
         __syncthreads();
     }
@@ -765,6 +769,14 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
 
     int consumed = 0;
     refill(0);
+    if (p.test_stall_ns > 0 && issued > 0 &&
+        !__all_sync(kFull, mbar_wait(smem_addr(&stall_bar), 0u, (unsigned long long)p.test_stall_ns))) {
+        // Injected stall: handled like a wait that ran out below, before any
+        // tile is consumed.
+        if (lane == 0) atomicOr(status, kFlagTimeout);
+        for (int k = 0; k < issued; ++k) mbar_wait(smem_addr(&wbars[k % kStages]), (uint32_t)((k / kStages) & 1));
+        consumed = issued;
+    }
     while (consumed < issued) {
         const int slot = consumed % kStages;
         const bool arrived = mbar_wait(smem_addr(&wbars[slot]), (uint32_t)((consumed / kStages) & 1));
@@ -926,7 +938,10 @@ cudaError_t launch_decode(const DecodeParams &p, const CUtensorMap &tmK, const C
         attr_limit[dev].store(limit, std::memory_order_release);
     }
     if (smem_bytes > (size_t)limit) return cudaErrorInvalidValue;
-    ps_decode_kernel<<<grid_ctas, kWorkersPerCta * 32, smem_bytes, stream>>>(p, tmK, tmV);
+    if ((e = take_injected_launch_error()) != cudaSuccess) return e;
+    DecodeParams q = p;
+    q.test_stall_ns = take_injected_stall_ns();
+    ps_decode_kernel<<<grid_ctas, kWorkersPerCta * 32, smem_bytes, stream>>>(q, tmK, tmV);
     return cudaGetLastError();
 }
 

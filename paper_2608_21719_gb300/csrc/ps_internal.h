@@ -104,11 +104,18 @@ struct DecodeParams {
     // K and V, bf16 [S][Hkv][128], written into its cache slot and attended.
     const uint16_t *k_new, *v_new;
     uint16_t *k_cache_w, *v_cache_w;
+    long long test_stall_ns;    // > 0: injected stall (ps_test_inject), else 0
 };
 
 // Launcher (ps_decode_kernels.cu).  Returns cudaSuccess or the launch error.
 // Adds one to the library's launch counter (ps_decode_launch_count()).
 void note_launch();
+
+// One-shot faults set by ps_test_inject(): the CUDA error the next launch
+// reports instead of launching (cudaSuccess: none), and the stall the next
+// decode launch makes (0: none).  Each call consumes what it returns.
+cudaError_t take_injected_launch_error();
+long long take_injected_stall_ns();
 
 cudaError_t launch_decode(const DecodeParams &p, const CUtensorMap &tmK, const CUtensorMap &tmV, int grid_ctas,
                           size_t smem_bytes, cudaStream_t stream);

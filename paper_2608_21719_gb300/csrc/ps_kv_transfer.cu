@@ -167,6 +167,7 @@ ps_status_t launch_xfer(const XferParams &xp, void *stream) {
         cudaFuncSetAttribute(ps_kv_transfer_kernel<kPack>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
             cudaSuccess)
         return PS_ERR_CUDA;
+    if (ps::take_injected_launch_error() != cudaSuccess) return PS_ERR_CUDA;
     ps_kv_transfer_kernel<kPack><<<sms * kXferCtasPerSm, kXferWarps * 32, smem, reinterpret_cast<cudaStream_t>(stream)>>>(xp);
     if (cudaGetLastError() != cudaSuccess) return PS_ERR_CUDA;
     ps::note_launch();

@@ -654,6 +654,7 @@ extern "C" ps_status_t ps_prefill_attention(const void *q, const void *k_cache, 
     pp.num_blocks = num_blocks;
     pp.scale_log2 = scale * 1.4426950408889634f;
     const dim3 grid((unsigned)nqt, (unsigned)num_kv_heads, (unsigned)num_seqs);
+    if (ps::take_injected_launch_error() != cudaSuccess) return PS_ERR_CUDA;
     ps_prefill_kernel<<<grid, kThreads, kSmemBytes, reinterpret_cast<cudaStream_t>(stream)>>>(tmQ, tmK, tmV, pp);
     if (cudaGetLastError() != cudaSuccess) return PS_ERR_CUDA;
     ps::note_launch();

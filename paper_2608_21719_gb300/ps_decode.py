@@ -35,6 +35,8 @@ PS_ERR_CUDA = -5
 PS_DEVICE_TIMEOUT = 1
 PS_DEVICE_BAD_BLOCK = 2
 PS_DEVICE_LEN_CLAMPED = 4
+PS_INJECT_LAUNCH_ERROR = 1
+PS_INJECT_DECODE_STALL = 2
 
 
 class PsError(RuntimeError):
@@ -79,6 +81,7 @@ _SIGS = {
     "ps_prefill_attention": (_i, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _i, _i, _i, _i, _i, _i, _i, _i,
                                   ctypes.c_longlong, _f, _vp, _vp]),
     "ps_decode_launch_count": (ctypes.c_ulonglong, []),
+    "ps_test_inject": (_i, [_i, ctypes.c_longlong]),
     "ps_status_string": (ctypes.c_char_p, [_i]),
     "ps_decode_abi_version": (_i, []),
 }
@@ -125,6 +128,10 @@ def ps_decode_abi_version() -> int:
 
 def ps_decode_launch_count() -> int:
     return _lib.ps_decode_launch_count()
+
+
+def ps_test_inject(kind, value) -> None:
+    _check(_lib.ps_test_inject(int(kind), int(value)), "ps_test_inject")
 
 
 def ps_decode_plan_create(num_seqs, num_q_heads, num_kv_heads, head_dim, block_size, max_blocks_per_seq,

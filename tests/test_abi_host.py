@@ -21,7 +21,8 @@ def test_every_declared_symbol_is_exported():
                 "ps_decode_attention_planned", "ps_decode_append_attention_planned",
                 "ps_decode_plan_set_timing_events",
                 "ps_decode_plan_read_device_status", "ps_decode_launch_count", "ps_status_string",
-                "ps_decode_abi_version", "ps_decode_attention_noalloc", "ps_kv_pack", "ps_kv_unpack"}
+                "ps_decode_abi_version", "ps_decode_attention_noalloc", "ps_kv_pack", "ps_kv_unpack",
+                "ps_test_inject"}
     assert expected <= set(names)
     lib = ctypes.CDLL(psd.LIB_PATH)
     for n in names:
@@ -170,3 +171,16 @@ def test_kv_transfer_validates_on_the_host():
     with pytest.raises(psd.PsError) as ei:  # too many sequences
         psd.ps_kv_unpack(16, off, 16, 4, 16, 5000, 8, 128, 16, 100, 16, 16, None, None)
     assert ei.value.status == psd.PS_ERR_UNSUPPORTED
+
+
+def test_fault_injection_arguments():
+    for kind, value in [(0, 1), (3, 1), (psd.PS_INJECT_LAUNCH_ERROR, -1), (psd.PS_INJECT_LAUNCH_ERROR, 10001),
+                        (psd.PS_INJECT_DECODE_STALL, 999), (psd.PS_INJECT_DECODE_STALL, 2 * 10**9)]:
+        with pytest.raises(psd.PsError) as ei:
+            psd.ps_test_inject(kind, value)
+        assert ei.value.status == psd.PS_ERR_INVALID_ARG
+    # valid values, then cleared again so that nothing leaks into later calls
+    psd.ps_test_inject(psd.PS_INJECT_LAUNCH_ERROR, 1)
+    psd.ps_test_inject(psd.PS_INJECT_LAUNCH_ERROR, 0)
+    psd.ps_test_inject(psd.PS_INJECT_DECODE_STALL, 10**6)
+    psd.ps_test_inject(psd.PS_INJECT_DECODE_STALL, 0)
