@@ -12,8 +12,12 @@
 // 128 MMA rows: 128 / g consecutive query tokens times the g query heads of
 // group j (row = token * g + head), so every K/V tile staged in shared memory
 // serves the whole group.  Keys stream in tiles of 128 through shared-memory
-// rings; every 16-key chunk of a tile is one TMA box of a (block, kv-head) page
-// of the cache, addressed through the block table.
+// rings; every 16-key chunk of a tile comes from one (block, kv-head) page of
+// the cache, addressed through the block table: for K as two TMA boxes (its
+// 64-column halves, stored [half][key][64], the K-major layout Q K^T needs),
+// for V as one box holding both halves ([chunk][half][16][64]; V is the
+// MN-major operand of P V, whose 64-column groups may sit 2 KiB apart), which
+// halves V's copies per tile.
 //
 // Per key tile n (warp roles, 7 warps):
 //   warps 0, 6 TMA producers: Q once and K_n into a three-stage ring (warp 0),
@@ -135,6 +139,13 @@ __device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *tm,
         : "memory");
 }
 // The same with an L2 cache-policy hint (from createpolicy).
+__device__ __forceinline__ void tma_load_4d_hint(uint32_t dst, const CUtensorMap *tm, int c0, int c1, int c2, int c3,
+                                                 uint32_t bar, uint64_t policy) {
+    asm volatile("cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
+        " [%0], [%1, {%2, %3, %4, %5}], [%6], %7;" ::"r"(dst), "l"(reinterpret_cast<uint64_t>(tm)), "r"(c0), "r"(c1),
+        "r"(c2), "r"(c3), "r"(bar), "l"(policy) : "memory");
+}
+
 __device__ __forceinline__ void tma_load_3d_hint(uint32_t dst, const CUtensorMap *tm, int c0, int c1, int c2,
                                                  uint32_t bar, uint64_t policy) {
     asm volatile(
@@ -359,7 +370,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t ring = is_k ? sK : sV;
         const CUtensorMap *tm = is_k ? &tmK : &tmV;
         const int *bt_row = p.block_table + (size_t)s * p.max_blocks_per_seq;
-        const int half = (lane >> 3) & 1, c = lane & 7;  // lanes 0-15: 8 chunks x 2 halves
+        const int half = (lane >> 3) & 1, c = lane & 7;  // K: lanes 0-15, 8 chunks x 2 halves; V: lanes 0-7
         // Every K/V page is read by all query tiles of its (sequence, head):
         // ask L2 to keep it (evict last).
         uint64_t keep;
@@ -375,15 +386,20 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t full = is_k ? bar_kfull(st) : bar_vfull(st);
             if (lane == 0) mbar_expect_tx(full, (uint32_t)(nc * 2 * kChunk * 128));
             __syncwarp();
-            if (lane < 16 && c < nc) {
-                const int t0 = base + c * kChunk;
+            if (is_k ? (lane < 16 && c < nc) : (lane < nc)) {
+                const int cc = is_k ? c : lane;
+                const int t0 = base + cc * kChunk;
                 const int lb = t0 / p.block_size;
                 const int b = __ldg(bt_row + lb);
                 int page = -1;  // out of range: TMA fills zeros
                 if (b >= 0 && (long long)b < p.num_blocks) page = b * p.num_kv_heads + j;
                 else if (p.status && is_k) atomicOr(p.status, (unsigned)PS_DEVICE_BAD_BLOCK);
-                tma_load_3d_hint(ring + st * kTile + half * kHalf + c * (kChunk * 128), tm, half * 64,
-                                 t0 - lb * p.block_size, page, full, keep);
+                if (is_k)
+                    tma_load_3d_hint(ring + st * kTile + half * kHalf + cc * (kChunk * 128), tm, half * 64,
+                                     t0 - lb * p.block_size, page, full, keep);
+                else  // both 64-column halves of the chunk in one box: [half][16][64]
+                    tma_load_4d_hint(ring + st * kTile + cc * (2 * kChunk * 128), tm, 0, t0 - lb * p.block_size, 0,
+                                     page, full, keep);
             }
             issued = n + 1;
         }
@@ -427,7 +443,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const int nvec = (kKeys - valid) * 8;
                     for (int e = lane; e < 2 * nvec; e += 32) {
                         const int h = e / nvec, r = e - h * nvec;
-                        *reinterpret_cast<uint4 *>(v + h * kHalf + valid * 128 + r * 16) = make_uint4(0, 0, 0, 0);
+                        const int key = valid + (r >> 3);
+                        *reinterpret_cast<uint4 *>(v + (key >> 4) * (2 * kChunk * 128) + h * (kChunk * 128) +
+                                                   (key & 15) * 128 + (r & 7) * 16) = make_uint4(0, 0, 0, 0);
                     }
                     fence_proxy_async_smem();
                     __syncwarp();
@@ -438,7 +456,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const uint32_t pt = tmem + kColP + (m & 1) * (kKeys / 2);
 #pragma unroll
                     for (int kk = 0; kk < kKeys / 16; ++kk)
-                        umma_ts(tmem + kColO, pt + kk * 8, smem_desc(vb + kk * 2048, 16384, 1024), idO,
+                        umma_ts(tmem + kColO, pt + kk * 8, smem_desc(vb + kk * 4096, 2048, 1024), idO,
                                 (m > 0 || kk > 0) ? 1u : 0u);
                     umma_commit(bar_pfree(m & 1));
                     umma_commit(bar_vfree(st));
@@ -595,6 +613,21 @@ bool encode3d(CUtensorMap *tm, const void *base, cuuint64_t d1, cuuint64_t d2, c
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// V as [page][slot][half][64]: dims (64, slot, half, page) with the half
+// stride (128 B) inside the slot stride (256 B), so that one box {64, 16, 2}
+// lands as [half][16][64] (both halves of a 16-key chunk in one copy).
+bool encode_v4d(CUtensorMap *tm, const void *base, cuuint64_t bs, cuuint64_t pages) {
+    EncodeTiledFn fn = encoder();
+    if (!fn) return false;
+    cuuint64_t dims[4] = {64, bs, 2, pages};
+    cuuint64_t strides[3] = {(cuuint64_t)kD * 2, 64 * 2, bs * kD * 2};
+    cuuint32_t box[4] = {64, kChunk, 2, 1};
+    cuuint32_t estr[4] = {1, 1, 1, 1};
+    return fn(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(base), dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
 
 }  // namespace
@@ -627,7 +660,7 @@ extern "C" ps_status_t ps_prefill_attention(const void *q, const void *k_cache, 
     CUtensorMap tmQ, tmK, tmV;
     if (!encode3d(&tmQ, q, (cuuint64_t)num_q_heads, (cuuint64_t)total_q_tokens, (cuuint32_t)g, (cuuint32_t)tpt) ||
         !encode3d(&tmK, k_cache, (cuuint64_t)block_size, (cuuint64_t)(num_blocks * num_kv_heads), kChunk, 1) ||
-        !encode3d(&tmV, v_cache, (cuuint64_t)block_size, (cuuint64_t)(num_blocks * num_kv_heads), kChunk, 1))
+        !encode_v4d(&tmV, v_cache, (cuuint64_t)block_size, (cuuint64_t)(num_blocks * num_kv_heads)))
         return PS_ERR_CUDA;
     // The shared-memory limit is a per-device function attribute: set it for
     // the current device on every call (cheap), so that a process driving
