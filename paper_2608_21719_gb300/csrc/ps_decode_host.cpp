@@ -81,18 +81,19 @@ EncodeTiledFn encode_fn() {
     return fn;
 }
 
-// 3-D view of a paged cache: dim0 = head_dim (contiguous), dim1 = slot within
-// the block, dim2 = (block, kv-head) page.  A box of 64 dims x 16 slots x 1
-// page lands in shared memory as one 128-byte-swizzled half tile.
+// 4-D view of a paged cache: dim0 = 64 dims of a half row (contiguous), dim1 =
+// slot within the block (256-byte stride), dim2 = half of the row (128-byte
+// stride), dim3 = (block, kv-head) page.  A box of 64 dims x 16 slots x 2
+// halves x 1 page lands in shared memory as one 128-byte-swizzled tile laid
+// out [half][slot][64], so one copy fetches a 16-token tile of K or V.
 ps_status_t encode_cache_map(CUtensorMap *tm, const void *base, const ps_decode_plan *p) {
     EncodeTiledFn fn = encode_fn();
     if (!fn) return PS_ERR_CUDA;
-    cuuint64_t dims[3] = {(cuuint64_t)kHeadDim, (cuuint64_t)p->block_size,
-                          (cuuint64_t)p->num_blocks * (cuuint64_t)p->num_kv_heads};
-    cuuint64_t strides[2] = {(cuuint64_t)kHeadDim * 2, (cuuint64_t)p->block_size * kHeadDim * 2};
-    cuuint32_t box[3] = {64, (cuuint32_t)kTileTokens, 1};
-    cuuint32_t estr[3] = {1, 1, 1};
-    CUresult r = fn(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims, strides, box, estr,
+    cuuint64_t dims[4] = {64, (cuuint64_t)p->block_size, 2, (cuuint64_t)p->num_blocks * (cuuint64_t)p->num_kv_heads};
+    cuuint64_t strides[3] = {(cuuint64_t)kHeadDim * 2, 64 * 2, (cuuint64_t)p->block_size * kHeadDim * 2};
+    cuuint32_t box[4] = {64, (cuuint32_t)kTileTokens, 2, 1};
+    cuuint32_t estr[4] = {1, 1, 1, 1};
+    CUresult r = fn(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(base), dims, strides, box, estr,
                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS ? PS_OK : PS_ERR_CUDA;

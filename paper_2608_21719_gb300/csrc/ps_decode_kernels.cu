@@ -14,8 +14,9 @@
 // the lengths and the grid, so results are bit-deterministic.
 //
 // Streaming.  A worker walks its range tile by tile.  Each tile's K and V
-// page halves arrive by TMA (cp.async.bulk.tensor, 128-byte swizzle) in a
-// per-warp ring of shared-memory stages completed on mbarriers; each
+// arrive by TMA (cp.async.bulk.tensor, 128-byte swizzle, one box each,
+// stored [64-column half][token][64]) in a per-warp ring of shared-memory
+// stages completed on mbarriers; each
 // (block, kv-head) page is read once for all g query heads of its group.
 // Per tile the warp computes S^T = K Q^T and O^T += V^T P^T on the tensor
 // cores (mma.sync m16n8k16, bf16 in, fp32 accumulate: tokens fill M = 16,
@@ -99,12 +100,12 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity,
     return true;
 }
 
-__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *tm, int c0, int c1, int c2,
+__device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap *tm, int c0, int c1, int c2, int c3,
                                             uint32_t bar) {
     asm volatile(
-        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-        " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
-        "l"(reinterpret_cast<uint64_t>(tm)), "r"(c0), "r"(c1), "r"(c2), "r"(bar)
+        "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3, %4, %5}], [%6];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(tm)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(bar)
         : "memory");
 }
 
@@ -665,10 +666,8 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
             const uint32_t qbytes = nx_new ? (uint32_t)(g * kHeadDim * 2) : 0u;
             fence_proxy_async_smem();
             mbar_arrive_expect_tx(bar, kStageBytes + qbytes);
-            tma_load_3d(dst, &tmK, 0, tok0, row, bar);
-            tma_load_3d(dst + kHalfBytes, &tmK, 64, tok0, row, bar);
-            tma_load_3d(dst + kTileBytes, &tmV, 0, tok0, row, bar);
-            tma_load_3d(dst + kTileBytes + kHalfBytes, &tmV, 64, tok0, row, bar);
+            tma_load_4d(dst, &tmK, 0, tok0, 0, row, bar);
+            tma_load_4d(dst + kTileBytes, &tmV, 0, tok0, 0, row, bar);
             if (nx_new) {
                 const uint16_t *qsrc = p.q + ((size_t)nx_s * p.num_q_heads + (size_t)nx_h * g) * kHeadDim;
                 bulk_load(smem_addr(qslots + ((pieces_issued - 1) % kQSlots) * kQSlotBytes), qsrc, qbytes, bar);

@@ -74,17 +74,17 @@ EncodeTiledFn tiled_encoder() {
     return fn;
 }
 
-// Same 3-D view of a paged cache the planned path uses: dims (head_dim, slot,
-// block x kv-head), box 64 x 16 x 1, 128-byte swizzle.
+// Same 4-D view of a paged cache the planned path uses: dims (64, slot, half,
+// block x kv-head) with the half stride inside the slot stride, box
+// 64 x 16 x 2 x 1, 128-byte swizzle.
 bool encode_cache(CUtensorMap *tm, const void *base, int block_size, long long num_blocks, int num_kv_heads) {
     EncodeTiledFn fn = tiled_encoder();
     if (!fn) return false;
-    cuuint64_t dims[3] = {(cuuint64_t)ps::kHeadDim, (cuuint64_t)block_size,
-                          (cuuint64_t)num_blocks * (cuuint64_t)num_kv_heads};
-    cuuint64_t strides[2] = {(cuuint64_t)ps::kHeadDim * 2, (cuuint64_t)block_size * ps::kHeadDim * 2};
-    cuuint32_t box[3] = {64, (cuuint32_t)ps::kTileTokens, 1};
-    cuuint32_t estr[3] = {1, 1, 1};
-    return fn(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims, strides, box, estr,
+    cuuint64_t dims[4] = {64, (cuuint64_t)block_size, 2, (cuuint64_t)num_blocks * (cuuint64_t)num_kv_heads};
+    cuuint64_t strides[3] = {(cuuint64_t)ps::kHeadDim * 2, 64 * 2, (cuuint64_t)block_size * ps::kHeadDim * 2};
+    cuuint32_t box[4] = {64, (cuuint32_t)ps::kTileTokens, 2, 1};
+    cuuint32_t estr[4] = {1, 1, 1, 1};
+    return fn(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(base), dims, strides, box, estr,
               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
