@@ -109,11 +109,10 @@ def test_forced_splits(psd, max_workers, min_stages):
 
 
 @pytest.mark.parametrize("max_workers,min_stages", [(0, 1), (40, 1), (57, 2)])
-def test_split_with_ranges_of_boundary_units_only(psd, max_workers, min_stages):
-    # Each segment costs its tiles plus a fixed number of boundary units in
-    # the static split; with many empty and one-tile sequences and ranges of
-    # one or two units, some ranges hold boundary units only (no tiles) and
-    # others start right at a segment.
+def test_split_with_many_empty_and_one_tile_sequences(psd, max_workers, min_stages):
+    # Ranges of one or two tiles (too short for the boundary weight: the
+    # plain equal split) over many empty and one-tile sequences, so that
+    # ranges start and end right at segments and cut one-tile segments.
     lengths = [0, 1, 0, 0, 16, 17, 0, 3, 33, 0, 1, 48, 0, 0, 5, 250, 0, 1, 1, 1]
     wl = _custom(16, 4, 16, lengths, seed=21, spare=9)
     out, status, info = _gpu(psd, wl, max_workers=max_workers, min_stages_per_worker=min_stages)
@@ -122,6 +121,19 @@ def test_split_with_ranges_of_boundary_units_only(psd, max_workers, min_stages):
     for s, L in enumerate(lengths):
         if L == 0:
             assert torch.all(out[s] == 0)
+
+
+def test_weighted_split_with_a_run_of_empty_sequences(psd):
+    # Long ranges (about 35 units each), so segment boundaries are weighted
+    # in the split, and a run of 20 empty sequences (4 boundary units per
+    # head each) long enough to hold whole ranges without a tile; short
+    # sequences in between.
+    lengths = [4096] * 8 + [0] * 20 + [4096] * 8 + [1, 17, 300] + [4096] * 4
+    wl = _custom(32, 8, 16, lengths, seed=23, spare=3)
+    out, status, info = _gpu(psd, wl)
+    assert status == 0
+    _compare(out, _oracle(wl), "weighted split with empty run", rel=0.0)
+    assert torch.all(out[8:28] == 0)
 
 
 def test_maximum_number_of_sequences(psd):
