@@ -305,9 +305,15 @@ ps_status_t ps_decode_plan_read_device_status(ps_decode_plan_t *plan, void *stre
  * num_blocks (physical blocks in k_cache / v_cache).  The work is split
  * statically, with the same kernel and the same numerics as the planned path.
  *
- * - The first call on each device resolves the device address of the scratch
- *   array (and sets the kernel's shared-memory limit) on that device; make
- *   that first call before any stream capture.
+ * - Every call looks up the scratch array's device address in the current
+ *   context, so a call after cudaDeviceReset() or under another context uses
+ *   that context's copy.  The first call on each device does the set-up:
+ *   under CUDA's default lazy module loading it loads the library's module
+ *   there, which commits the array's PS_NOALLOC_SCRATCH_BYTES of device
+ *   memory at that moment, and it sets the kernel's shared-memory limit.  A
+ *   server that forbids allocation after start-up should therefore make one
+ *   call on each device during start-up (or set CUDA_MODULE_LOADING=EAGER),
+ *   and that first call must come before any stream capture.
  * - Every call shares the one array and first clears its counters on
  *   `stream`.  Calls that overlap on the GPU (other streams, other host
  *   threads) race on the array and produce wrong results: serialise them.

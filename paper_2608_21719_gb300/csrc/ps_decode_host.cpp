@@ -44,25 +44,6 @@ bool live(const ps_decode_plan *p) { return p != nullptr && p->magic == kPlanMag
 
 bool aligned(const void *p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
 
-ps_status_t check_shape(int num_seqs, int num_q_heads, int num_kv_heads, int head_dim, int block_size,
-                        int max_blocks_per_seq, long long num_blocks) {
-    if (num_seqs <= 0 || num_q_heads <= 0 || num_kv_heads <= 0 || head_dim <= 0 || block_size <= 0 ||
-        max_blocks_per_seq <= 0 || num_blocks <= 0)
-        return PS_ERR_INVALID_ARG;
-    if (num_q_heads % num_kv_heads != 0) return PS_ERR_INVALID_ARG;
-    if (head_dim != kHeadDim) return PS_ERR_UNSUPPORTED;
-    if (num_q_heads / num_kv_heads > kMaxGroup) return PS_ERR_UNSUPPORTED;
-    if (block_size % kTileTokens != 0 || block_size > 256) return PS_ERR_UNSUPPORTED;
-    if (num_seqs > kMaxSeqs || partial_smem_bytes(num_seqs) > kMaxSmemPerCta) return PS_ERR_UNSUPPORTED;
-    // Tile counts, the split's cost units and TMA row coordinates are 32-bit.
-    const long long len_cap = (long long)max_blocks_per_seq * block_size;
-    const long long tiles = (long long)num_seqs * ((len_cap + kTileTokens - 1) / kTileTokens) * num_kv_heads;
-    const long long units = tiles + (long long)kSegmentCost * num_kv_heads * num_seqs;
-    if (len_cap > INT32_MAX || units > INT32_MAX) return PS_ERR_UNSUPPORTED;
-    if (num_blocks * num_kv_heads > INT32_MAX) return PS_ERR_UNSUPPORTED;
-    return PS_OK;
-}
-
 using EncodeTiledFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
                                    const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
                                    CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
@@ -202,7 +183,7 @@ ps_status_t ps_decode_plan_create_ex(int num_seqs, int num_q_heads, int num_kv_h
     *workspace_bytes = 0;
     if (num_sms < 0 || max_workers < 0 || min_stages_per_worker < 0) return PS_ERR_INVALID_ARG;
     if (num_sms > kMaxGridCtas) return PS_ERR_UNSUPPORTED;
-    ps_status_t e = check_shape(num_seqs, num_q_heads, num_kv_heads, head_dim, block_size, max_blocks_per_seq,
+    ps_status_t e = check_decode_shape(num_seqs, num_q_heads, num_kv_heads, head_dim, block_size, max_blocks_per_seq,
                                 num_blocks);
     if (e != PS_OK) return e;
     if (num_sms == 0) {

@@ -34,25 +34,18 @@ constexpr size_t kNoallocScratchBytes = (size_t)PS_NOALLOC_SCRATCH_BYTES;
 // cudaGetSymbolAddress() below.
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoallocScratchBytes];
 
-constexpr int kMaxDevices = 64;
-std::mutex g_setup_mu;
-void *g_scratch_ptr[kMaxDevices] = {};
-
-// Device address of the scratch array on the current device, resolved once per
-// device (with that device current) on the first call made on it.
+// Device address of the scratch array in the current context.  It is
+// resolved on every call rather than cached: the address belongs to the
+// context, and after cudaDeviceReset() (or with another context current) a
+// cached one would point at memory that is no longer this array's.  The
+// lookup is cheap next to the launch.  Under lazy module loading (the CUDA
+// default) the first lookup on a device is also what loads this module and
+// commits the array's memory on that device.
 cudaError_t scratch_address(void **out) {
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
+    void *ptr = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&ptr, g_noalloc_scratch);
     if (e != cudaSuccess) return e;
-    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
-    std::lock_guard<std::mutex> lk(g_setup_mu);
-    if (g_scratch_ptr[dev] == nullptr) {
-        void *ptr = nullptr;
-        e = cudaGetSymbolAddress(&ptr, g_noalloc_scratch);
-        if (e != cudaSuccess) return e;
-        g_scratch_ptr[dev] = ptr;
-    }
-    *out = g_scratch_ptr[dev];
+    *out = ptr;
     return cudaSuccess;
 }
 
@@ -103,30 +96,24 @@ extern "C" ps_status_t ps_decode_attention_noalloc(const void *q, const void *k_
     if (!is_aligned(q, 16) || !is_aligned(k_cache, 16) || !is_aligned(v_cache, 16) || !is_aligned(out, 16) ||
         !is_aligned(block_table, 4) || !is_aligned(seq_lens, 4))
         return PS_ERR_INVALID_ARG;
-    if (num_seqs <= 0 || num_q_heads <= 0 || num_kv_heads <= 0 || head_dim <= 0 || block_size <= 0 ||
-        max_blocks_per_seq <= 0 || num_blocks <= 0 || num_q_heads % num_kv_heads != 0 || !std::isfinite(scale))
-        return PS_ERR_INVALID_ARG;
-    if (head_dim != kHeadDim || num_q_heads / num_kv_heads > kMaxGroup || block_size % kTileTokens != 0 ||
-        block_size > 256 || num_seqs > kMaxSeqs || partial_smem_bytes(num_seqs) > kMaxSmemPerCta)
-        return PS_ERR_UNSUPPORTED;
+    if (!std::isfinite(scale)) return PS_ERR_INVALID_ARG;
+    // The same shape check as the planned path (supported set and the 32-bit
+    // bounds of the device split).
+    const ps_status_t shape = check_decode_shape(num_seqs, num_q_heads, num_kv_heads, head_dim, block_size,
+                                                 max_blocks_per_seq, num_blocks);
+    if (shape != PS_OK) return shape;
     const long long len_cap = (long long)max_blocks_per_seq * block_size;
-    if (len_cap > INT32_MAX || (long long)num_seqs * ((len_cap + kTileTokens - 1) / kTileTokens) * num_kv_heads > INT32_MAX ||
-        num_blocks * num_kv_heads > INT32_MAX)
-        return PS_ERR_UNSUPPORTED;
 
+    // The per-segment counters alone may already exceed the array.
+    if (kWsHeaderBytes + (size_t)num_seqs * num_kv_heads * 4 > kNoallocScratchBytes) return PS_ERR_UNSUPPORTED;
     int dev = 0, sms = 0;
     if (cudaGetDevice(&dev) != cudaSuccess ||
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0)
         return PS_ERR_CUDA;
-    // Scratch layout: header, per-segment counters, then two partial slots per
-    // worker range, the layout the planned path uses.
-    const int workers = sms * kWorkersPerCta;
-    const size_t seg_off = kWsHeaderBytes;
-    const size_t acc_off = align_up(seg_off + (size_t)num_seqs * num_kv_heads * 4, 256);
-    const size_t slots = 2 * (size_t)workers;
-    const size_t ml_off = align_up(acc_off + slots * kSlotFloats * 4, 256);
-    const size_t need = align_up(ml_off + slots * kSlotMl * 4, 256);
-    if (need > kNoallocScratchBytes) return PS_ERR_UNSUPPORTED;  // beyond the fixed scratch array
+    // Scratch layout: the planned path's workspace layout (header,
+    // per-segment counters, two partial slots per worker range).
+    const WorkspaceLayout lay = workspace_layout(num_seqs, num_kv_heads, sms * kWorkersPerCta);
+    if (lay.total > kNoallocScratchBytes) return PS_ERR_UNSUPPORTED;  // beyond the fixed scratch array
 
     void *scratch = nullptr;
     if (scratch_address(&scratch) != cudaSuccess) return PS_ERR_CUDA;
@@ -139,7 +126,7 @@ extern "C" ps_status_t ps_decode_attention_noalloc(const void *q, const void *k_
     uint8_t *ws = static_cast<uint8_t *>(scratch);
     // Counters and the status word must start at zero; the previous call's
     // contents are still in the array.
-    if (cudaMemsetAsync(ws, 0, acc_off, st) != cudaSuccess) return PS_ERR_CUDA;
+    if (cudaMemsetAsync(ws, 0, lay.acc_off, st) != cudaSuccess) return PS_ERR_CUDA;
 
     DecodeParams dp;
     dp.q = static_cast<const uint16_t *>(q);
@@ -147,9 +134,9 @@ extern "C" ps_status_t ps_decode_attention_noalloc(const void *q, const void *k_
     dp.seq_lens = seq_lens;
     dp.out = static_cast<uint16_t *>(out);
     dp.ws_header = reinterpret_cast<int *>(ws);
-    dp.seg_done = reinterpret_cast<int *>(ws + seg_off);
-    dp.ws_acc = reinterpret_cast<float *>(ws + acc_off);
-    dp.ws_ml = reinterpret_cast<float *>(ws + ml_off);
+    dp.seg_done = reinterpret_cast<int *>(ws + lay.seg_done_off);
+    dp.ws_acc = reinterpret_cast<float *>(ws + lay.acc_off);
+    dp.ws_ml = reinterpret_cast<float *>(ws + lay.ml_off);
     dp.num_seqs = num_seqs;
     dp.num_q_heads = num_q_heads;
     dp.num_kv_heads = num_kv_heads;
@@ -158,7 +145,7 @@ extern "C" ps_status_t ps_decode_attention_noalloc(const void *q, const void *k_
     dp.max_blocks_per_seq = max_blocks_per_seq;
     dp.num_blocks = num_blocks;
     dp.len_cap = (int)len_cap;
-    dp.max_workers = workers;
+    dp.max_workers = sms * kWorkersPerCta;
     dp.min_stages = kDefaultMinStages;
     dp.scale_log2 = (float)((double)scale * 1.4426950408889634);
     dp.k_new = dp.v_new = nullptr;

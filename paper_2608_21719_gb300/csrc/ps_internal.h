@@ -8,6 +8,8 @@
 #include <stddef.h>
 #include <stdint.h>
 
+#include "ps_decode.h"
+
 namespace ps {
 
 // Shapes the kernel is written for.
@@ -83,6 +85,29 @@ constexpr size_t kMaxSmemPerCta = 227 * 1024;  // opt-in limit of one CTA on sm_
 inline size_t partial_smem_bytes(int num_seqs) {
     return 1024 /* alignment slack */ + (size_t)kWorkersPerCta * kWorkerBytes +
            (size_t)kWorkersPerCta * (kStages * (8 + 16) + 4 * 16) + (size_t)(2 * num_seqs + 1) * 4;
+}
+
+// Host-side shape check shared by every decode entry point (planned and
+// workspace-free), so that both reject exactly the same shapes.  Besides the
+// supported set it bounds what the device split computes in 32 bits: tile
+// counts, the split's cost units (tiles plus kSegmentCost per segment
+// boundary, Partition::seq_unit) and TMA row coordinates.
+inline ps_status_t check_decode_shape(int num_seqs, int num_q_heads, int num_kv_heads, int head_dim,
+                                      int block_size, int max_blocks_per_seq, long long num_blocks) {
+    if (num_seqs <= 0 || num_q_heads <= 0 || num_kv_heads <= 0 || head_dim <= 0 || block_size <= 0 ||
+        max_blocks_per_seq <= 0 || num_blocks <= 0)
+        return PS_ERR_INVALID_ARG;
+    if (num_q_heads % num_kv_heads != 0) return PS_ERR_INVALID_ARG;
+    if (head_dim != kHeadDim) return PS_ERR_UNSUPPORTED;
+    if (num_q_heads / num_kv_heads > kMaxGroup) return PS_ERR_UNSUPPORTED;
+    if (block_size % kTileTokens != 0 || block_size > 256) return PS_ERR_UNSUPPORTED;
+    if (num_seqs > kMaxSeqs || partial_smem_bytes(num_seqs) > kMaxSmemPerCta) return PS_ERR_UNSUPPORTED;
+    const long long len_cap = (long long)max_blocks_per_seq * block_size;
+    const long long tiles = (long long)num_seqs * ((len_cap + kTileTokens - 1) / kTileTokens) * num_kv_heads;
+    const long long units = tiles + (long long)kSegmentCost * num_kv_heads * num_seqs;
+    if (len_cap > INT32_MAX || units > INT32_MAX) return PS_ERR_UNSUPPORTED;
+    if (num_blocks * num_kv_heads > INT32_MAX) return PS_ERR_UNSUPPORTED;
+    return PS_OK;
 }
 
 struct DecodeParams {

@@ -29,6 +29,12 @@ def test_every_declared_symbol_is_exported():
         assert hasattr(lib, n), n
 
 
+def test_binding_constants_match_the_header():
+    text = open(psd.HEADER_PATH).read()
+    assert "#define PS_NOALLOC_SCRATCH_BYTES (16u << 20)" in text
+    assert psd.PS_NOALLOC_SCRATCH_BYTES == 16 << 20
+
+
 def test_status_strings_and_version():
     assert psd.ps_status_string(0) == "ok"
     for s in (-1, -2, -3, -4, -5):
@@ -88,6 +94,38 @@ def test_plan_rejects_bad_shapes(kw, status):
     with pytest.raises(psd.PsError) as ei:
         _plan(**kw)
     assert ei.value.status == status
+
+
+def test_noalloc_rejects_what_the_planned_path_rejects():
+    """The workspace-free entry point applies the planned path's shape check,
+    including the 32-bit bound on the split's cost units: 4096 sequences x 8
+    kv heads x 65535 tiles stay below 2^31 tiles, but the boundary weight of
+    the 32768 segments pushes the units past it.  Both entry points reject
+    it before any CUDA call."""
+    S, Hkv, mbps = 4096, 8, 65535
+    tiles = S * Hkv * mbps
+    assert tiles < 2**31 <= tiles + 4 * Hkv * S
+    with pytest.raises(psd.PsError) as ei:
+        _plan(num_seqs=S, num_q_heads=8 * Hkv, num_kv_heads=Hkv, max_blocks_per_seq=mbps)
+    assert ei.value.status == psd.PS_ERR_UNSUPPORTED
+    with pytest.raises(psd.PsError) as ei:
+        psd.ps_decode_attention_noalloc(256, 256, 256, 256, 256, 256, S, 8 * Hkv, Hkv, 128, 16, mbps, 1, 0.1, None)
+    assert ei.value.status == psd.PS_ERR_UNSUPPORTED
+    # The rest of the shared check: bad group, block size, head_dim, sequence count.
+    for args, status in [((8, 3, 128, 16), psd.PS_ERR_INVALID_ARG), ((8, 2, 128, 8), psd.PS_ERR_UNSUPPORTED),
+                         ((8, 2, 64, 16), psd.PS_ERR_UNSUPPORTED), ((128, 8, 128, 16), psd.PS_ERR_UNSUPPORTED)]:
+        Hq, Hk, d, bs = args
+        with pytest.raises(psd.PsError) as ei:
+            psd.ps_decode_attention_noalloc(256, 256, 256, 256, 256, 256, 4, Hq, Hk, d, bs, 8, 100, 0.1, None)
+        assert ei.value.status == status
+    with pytest.raises(psd.PsError) as ei:
+        psd.ps_decode_attention_noalloc(256, 256, 256, 256, 256, 256, 4097, 8, 2, 128, 16, 8, 100, 0.1, None)
+    assert ei.value.status == psd.PS_ERR_UNSUPPORTED
+    # Counters alone beyond the fixed array: 4096 sequences x 1025 kv heads x 4 bytes.
+    assert 4096 * 1025 * 4 > psd.PS_NOALLOC_SCRATCH_BYTES
+    with pytest.raises(psd.PsError) as ei:
+        psd.ps_decode_attention_noalloc(256, 256, 256, 256, 256, 256, 4096, 1025, 1025, 128, 16, 1, 16, 0.1, None)
+    assert ei.value.status == psd.PS_ERR_UNSUPPORTED
 
 
 def test_calls_validate_before_touching_the_device():

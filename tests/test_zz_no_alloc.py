@@ -6,12 +6,16 @@ tensors it passes, a server that forbids allocation after start-up -- call
 ps_decode_attention_noalloc, whose split-KV scratch is a fixed device array
 inside the library.  These tests call it through the C ABI and check it
 against the planned entry point, twice in a row, since the array keeps the
-previous call's contents.  This file is collected last on purpose.
+previous call's contents.  The split is the planned path's default one
+(every streaming warp, the default minimum share), so the output must be
+bit-identical to the planned call's; it is also held to the fp64 oracle's
+bounds.  This file is collected last on purpose.
 """
 import numpy as np
 import pytest
 import torch
 
+import oracle
 from paper_2608_21719_gb300 import inputs
 
 pytestmark = pytest.mark.gpu
@@ -41,7 +45,6 @@ def _workload(Hq, Hkv, bs, lengths, seed):
 
 def _close(got, ref):
     got = got.float().cpu().numpy().astype(np.float64)
-    ref = ref.float().cpu().numpy().astype(np.float64)
     assert np.all(np.isfinite(got))
     err = np.abs(got - ref)
     assert np.all(err <= MAX_ABS + BF16_REL * np.abs(ref)), "max abs err %.3g" % err.max()
@@ -55,6 +58,9 @@ def _close(got, ref):
 ])
 def test_noalloc_matches_planned_path_on_consecutive_calls(psd, case):
     wl = _workload(case["Hq"], case["Hkv"], case["bs"], case["lengths"], case["seed"])
+    want = oracle.decode_attention(inputs.bf16_bits(wl.q), inputs.bf16_bits(wl.k_cache),
+                                   inputs.bf16_bits(wl.v_cache), wl.block_table.cpu().numpy(),
+                                   wl.seq_lens.cpu().numpy(), wl.num_kv_heads, wl.scale)
     attn = psd.DecodeAttention.for_workload(wl)
     ref = attn(wl.q, wl.k_cache, wl.v_cache, wl.block_table, wl.seq_lens, scale=wl.scale)
     torch.cuda.synchronize()
@@ -66,13 +72,16 @@ def test_noalloc_matches_planned_path_on_consecutive_calls(psd, case):
                                         wl.num_seqs, wl.num_q_heads, wl.num_kv_heads, 128, wl.block_size,
                                         wl.max_blocks_per_seq, wl.num_blocks, wl.scale, stream)
         torch.cuda.synchronize()
-        _close(out, ref)
+        assert torch.equal(out, ref)
+        _close(out, want)
 
 
 def test_noalloc_rejects_shapes_beyond_its_scratch(psd):
-    # 4096 sequences x 512 kv heads need 8 MiB of per-segment counters on top
-    # of the partial slots: more than the fixed array holds.
+    # 4096 sequences x 1025 kv heads need 16.8 MB of per-segment counters
+    # alone, more than the fixed array holds whatever the SM count, so the
+    # call is rejected before anything is launched.
+    assert 256 + 4096 * 1025 * 4 > psd.PS_NOALLOC_SCRATCH_BYTES
     t = torch.zeros(64, dtype=torch.int32, device="cuda")
     with pytest.raises(psd.PsError) as ei:
-        psd.ps_decode_attention_noalloc(t, t, t, t, t, t, 4096, 512, 512, 128, 16, 1, 16, 0.1, None)
+        psd.ps_decode_attention_noalloc(t, t, t, t, t, t, 4096, 1025, 1025, 128, 16, 1, 16, 0.1, None)
     assert ei.value.status == psd.PS_ERR_UNSUPPORTED
