@@ -110,31 +110,23 @@ def test_single_token_append_returns_the_new_value(psd):
             assert torch.equal(out[s, h], v_new[s, h // 4])
 
 
-def test_append_at_full_size_sampled(psd):
+def test_append_at_full_size_every_output(psd):
+    """The Llama-3-8B-shaped batch at full size: every output against the
+    oracle on the host-appended cache, and the whole cache bit-for-bit."""
     wl = inputs.make_workload(2, device="cuda", poison=False)
     gen = torch.Generator(device="cuda").manual_seed(1234)
     k_new = torch.randn((wl.num_seqs, wl.num_kv_heads, 128), generator=gen, device="cuda").to(torch.bfloat16)
     v_new = torch.randn((wl.num_seqs, wl.num_kv_heads, 128), generator=gen, device="cuda").to(torch.bfloat16)
+    host = inputs.Workload(cfg=None, q=wl.q.cpu(), k_cache=wl.k_cache.cpu(), v_cache=wl.v_cache.cpu(),
+                           block_table=wl.block_table.cpu(), seq_lens=wl.seq_lens.cpu(), scale=wl.scale)
+    k_ref, v_ref = _host_append(host, k_new.cpu(), v_new.cpu())
     attn = psd.DecodeAttention.for_workload(wl)
     out = attn.append(wl.q, k_new, v_new, wl.k_cache, wl.v_cache, wl.block_table, wl.seq_lens, scale=wl.scale)
     torch.cuda.synchronize()
+    assert attn.device_status() == 0
     attn.close()
-    lens = wl.seq_lens.cpu().numpy()
-    bs = wl.block_size
-    idx = sorted({int(np.argmin(lens)), int(np.argmax(lens)), 0, 17, 40})
-    for s in idx:  # the cache slot of the new token now holds k_new / v_new
-        L = int(lens[s])
-        b = int(wl.block_table[s, (L - 1) // bs])
-        assert torch.equal(wl.k_cache[b, :, (L - 1) % bs], k_new[s])
-        assert torch.equal(wl.v_cache[b, :, (L - 1) % bs], v_new[s])
-    pages = [wl.block_table[s, :(int(lens[s]) + bs - 1) // bs].cpu().numpy() for s in idx]
-    flat = torch.from_numpy(np.concatenate(pages).astype(np.int64)).cuda()
-    nbt = np.full((len(idx), max(len(p) for p in pages)), -1, dtype=np.int32)
-    pos = 0
-    for i, pg in enumerate(pages):
-        nbt[i, :len(pg)] = np.arange(pos, pos + len(pg))
-        pos += len(pg)
-    ref = oracle.decode_attention(inputs.bf16_bits(wl.q[idx]), inputs.bf16_bits(wl.k_cache.index_select(0, flat)),
-                                  inputs.bf16_bits(wl.v_cache.index_select(0, flat)), nbt, lens[idx],
-                                  wl.num_kv_heads, wl.scale)
-    _check(out[idx].cpu(), ref, rel=0.0)
+    assert torch.equal(wl.k_cache.cpu().view(torch.int16), k_ref.view(torch.int16))
+    assert torch.equal(wl.v_cache.cpu().view(torch.int16), v_ref.view(torch.int16))
+    ref = oracle.decode_attention(inputs.bf16_bits(host.q), inputs.bf16_bits(k_ref), inputs.bf16_bits(v_ref),
+                                  host.block_table.numpy(), host.seq_lens.numpy(), wl.num_kv_heads, wl.scale)
+    _check(out.cpu(), ref, rel=0.0)
