@@ -9,10 +9,15 @@ written and read back, so that no dirty lines are written back inside the
 next step), and each step is timed with CUDA events on the launching
 stream.
 
-Prints one JSON line.  Default workload: the Llama-3-8B-shaped decode layer
-(64 sequences, 32/8 heads, block 16, contexts U[1024, 4096]).  --config
-picks another of the five workloads.  --impl reference times the fp64 CPU
-oracle on the host cores instead (bounded samples of the same workload).
+Prints one JSON line.  By default the four large workloads run one after
+another in this process, each timed for --steps steps: the headline
+(value, roofline, e2e, cpu_baseline, clocks) is the largest single-GPU
+workload, the 70B-shaped 256-sequence batch (block 32, contexts
+U[2048, 8192] in a 6 GiB pool); the Llama-3-8B, long-thinking and
+mixed-phase batches follow under "per_config", each with its own roofline
+fraction, e2e figure and clock record.  --config k times workload k alone.
+--impl reference times the fp64 CPU oracle on the host cores instead
+(bounded samples of the same workload).
 
 Multi-GPU (torchrun, one process per GPU): every rank runs its own batch of
 the workload (weak scaling, no collective on the data path); the value is
@@ -40,12 +45,14 @@ FALLBACK_HBM_GBS = 6800.0
 NOMINAL_HBM_GBS = 7900.0  # NVIDIA's GB300 HBM3e figure, for a labelled second fraction only
 # Layers of the model each workload is shaped after (8B: 32, 32B: 64, 70B: 80).
 MODEL_LAYERS = {1: None, 2: 32, 3: 32, 4: 64, 5: 80}
-PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "ps_decode_kernel_llama3-8b-decode.md")
+PROFILES = os.path.join(ROOT, "profiles")
+HEADLINE_CONFIG = 5            # the largest workload that fits one GPU
+DEFAULT_CONFIGS = (5, 2, 3, 4)  # headline first, then the other large workloads
 PREFILL_SUMMARY = os.path.join(ROOT, "profiles", "ps_prefill_kernel_llama3-8b-chunked-prefill.md")
 PREFILL_SOURCE = os.path.join(ROOT, "paper_2608_21719_gb300", "csrc", "ps_prefill.cu")
 FALLBACK_BF16_TFLOPS = 1900.0
 KERNEL_SOURCE = os.path.join(ROOT, "paper_2608_21719_gb300", "csrc", "ps_decode_kernels.cu")
-CLOCK_QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+CLOCK_QUERY = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
                "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
                "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
@@ -56,7 +63,8 @@ def parse_args(argv=None):
     ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--config", type=int, default=2, choices=[1, 2, 3, 4, 5])
+    ap.add_argument("--config", type=int, default=None, choices=[1, 2, 3, 4, 5],
+                    help="time this workload alone (default: workloads 5, 2, 3, 4, headline 5)")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="CPU time budget of the oracle baseline sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -112,9 +120,16 @@ def measured_peaks():
         return FALLBACK_HBM_GBS, "fallback"
 
 
-def profiled_traffic(summary=PROFILE_SUMMARY, source=KERNEL_SOURCE):
-    """Per-launch DRAM bytes of a kernel from its committed ncu summary, or
-    None when the kernel source changed since it was taken."""
+def decode_profile_summary(workload: str) -> str:
+    """Path of the committed ncu summary of the decode kernel on a workload."""
+    return os.path.join(PROFILES, "ps_decode_kernel_%s.md" % workload)
+
+
+def profiled_traffic(summary, source=KERNEL_SOURCE, workload=None):
+    """Per-launch DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum)
+    of a kernel from its committed ncu summary of this workload, or None
+    when there is no summary for it, it names another workload, or the
+    kernel source changed since the counters were taken."""
     try:
         text = open(summary).read()
         src_hash = hashlib.sha256(open(source, "rb").read()).hexdigest()
@@ -128,6 +143,8 @@ def profiled_traffic(summary=PROFILE_SUMMARY, source=KERNEL_SOURCE):
             vals[k.strip().strip("`")] = v.strip().strip("`")
     if vals.get("kernel_source_sha256") != src_hash:
         return None
+    if workload is not None and vals.get("workload") != workload:
+        return None
     try:
         return int(float(vals["traffic_bytes_per_launch"]))
     except (KeyError, ValueError):
@@ -135,12 +152,19 @@ def profiled_traffic(summary=PROFILE_SUMMARY, source=KERNEL_SOURCE):
 
 
 class ClockSampler:
-    """nvidia-smi sampling of SM clocks and throttle reasons during the timed region."""
+    """nvidia-smi sampling (read-only queries) of SM clocks and throttle
+    reasons, polled every 5 ms.  mark_start()/mark_end() bracket the timed
+    region on the host clock; the summary counts the samples whose
+    nvidia-smi timestamps fall inside it (falling back to all samples taken
+    while the sampler ran when the region is shorter than one poll)."""
 
-    def __init__(self, gpu_index: int):
+    POLL_MS = 5
+
+    def __init__(self, gpu_index):
         self.gpu = gpu_index
         self.proc = None
         self.path = None
+        self.t0 = self.t1 = None
 
     def __enter__(self):
         fd, self.path = tempfile.mkstemp(prefix="ps_clocks_", suffix=".csv")
@@ -148,13 +172,20 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.gpu), "--query-gpu=" + CLOCK_QUERY, "--format=csv,noheader,nounits",
-                 "-lms", "100"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+                 "-lms", str(self.POLL_MS)], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
         except (OSError, FileNotFoundError):
             self.proc = None
-        time.sleep(0.15)
+        time.sleep(0.3)
         return self
 
+    def mark_start(self):
+        self.t0 = time.time()
+
+    def mark_end(self):
+        self.t1 = time.time()
+
     def __exit__(self, *exc):
+        time.sleep(0.05)
         if self.proc is not None:
             self.proc.terminate()
             try:
@@ -162,29 +193,51 @@ class ClockSampler:
             except subprocess.TimeoutExpired:
                 self.proc.kill()
 
+    @staticmethod
+    def _stamp(text):
+        import datetime
+        for fmt in ("%Y/%m/%d %H:%M:%S.%f", "%Y/%m/%d %H:%M:%S"):
+            try:
+                return datetime.datetime.strptime(text.strip(), fmt).timestamp()
+            except ValueError:
+                continue
+        return None
+
     def summary(self):
         if self.proc is None or self.path is None:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
         rows = []
         for line in open(self.path):
             parts = [p.strip() for p in line.split(",")]
-            if len(parts) >= 9:
+            if len(parts) >= 10:
                 rows.append(parts)
         os.unlink(self.path)
         if not rows:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"], "samples": 0}
+
         def num(x):
             try:
                 return float(x)
             except ValueError:
                 return None
-        sm = [num(r[1]) for r in rows if num(r[1]) is not None]
-        mx = [num(r[2]) for r in rows if num(r[2]) is not None]
+        inside = rows
+        if self.t0 is not None and self.t1 is not None:
+            # nvidia-smi prints local wall-clock time; allow one poll of slack at each end.
+            slack = self.POLL_MS * 1e-3
+            sel = [r for r in rows if (lambda t: t is not None and self.t0 - slack <= t <= self.t1 + slack)(
+                self._stamp(r[0]))]
+            if sel:
+                inside = sel
+        sm = [num(r[2]) for r in inside if num(r[2]) is not None]
+        mx = [num(r[3]) for r in inside if num(r[3]) is not None]
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower() == "active"})
-        power = [num(r[3]) for r in rows if num(r[3]) is not None]
+        reasons = sorted({names[i] for r in inside for i in range(4) if r[6 + i].lower() == "active"})
+        power = [num(r[4]) for r in inside if num(r[4]) is not None]
         return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
-                "reasons": reasons, "samples": len(rows), "power_w_max": max(power) if power else None}
+                "reasons": reasons, "samples": len(inside), "samples_total": len(rows),
+                "in_region": inside is not rows, "poll_ms": self.POLL_MS,
+                "region_ms": None if self.t0 is None or self.t1 is None else round((self.t1 - self.t0) * 1e3, 2),
+                "power_w_max": max(power) if power else None}
 
 
 def sample_for_oracle(wl, seq_idx, token_cap=None):
@@ -251,19 +304,44 @@ def choose_oracle_sample(wl, budget_s, threads):
 
 # ------------------------------------------------------------- our arm ------
 
-def run_ours(args):
-    import numpy as np
+def workload_config(cfg, wl, alg, flush_mb, world, append=False):
+    """The "config" object of a bench line; both arms print the same one for
+    the same workload."""
+    lens = wl.seq_lens.cpu().numpy()
+    return {
+        "workload": cfg.name,
+        "num_seqs": wl.num_seqs, "num_q_heads": wl.num_q_heads, "num_kv_heads": wl.num_kv_heads,
+        "head_dim": wl.head_dim, "block_size": wl.block_size, "lengths": list(cfg.lengths),
+        "seed": cfg.seed, "total_tokens": int(lens.sum()), "kv_bytes": alg["kv"],
+        "pool_blocks": wl.num_blocks,
+        "l2": "flushed before every step, outside the timed interval: write then read of a %d MB buffer" % flush_mb,
+        "parallelism": "replicas" if world == 1 else "dp%d (independent batches per GPU)" % world,
+        "step": "append current token K/V + attend" if append else "attend",
+    }
+
+
+def flush_bytes(dev) -> int:
+    import torch
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    return max(2 * l2, 64 << 20) // 4 * 4
+
+
+def gpu_index_of(local_rank: int) -> str:
+    visible = [x.strip() for x in os.environ.get("CUDA_VISIBLE_DEVICES", "").split(",") if x.strip()]
+    return visible[local_rank] if local_rank < len(visible) else str(local_rank)
+
+
+def measure_decode(args, key, dev, rank, local_rank, world):
+    """Time one workload: kernel-only steps (CUDA events on the launching
+    stream, L2 flushed before each), then the end-to-end loop through the
+    public API with host buffers.  Returns (fields of the JSON line, the
+    workload, its algorithmic bytes) on every rank."""
     import torch
     import torch.distributed as dist
 
     from paper_2608_21719_gb300 import inputs, ps_decode, roofline
 
-    rank, local_rank, world = dist_env()
-    if world > 1 and not dist.is_initialized():
-        dist.init_process_group("nccl")
-    torch.cuda.set_device(local_rank)
-    dev = torch.device("cuda", local_rank)
-    cfg = inputs.CONFIGS[args.config]
+    cfg = inputs.CONFIGS[key]
     wl = inputs.make_workload(cfg, device=dev, poison=False)
     lens = wl.seq_lens.cpu().numpy()
     alg = roofline.algorithmic_bytes(lens, wl.num_q_heads, wl.num_kv_heads, wl.head_dim, wl.block_size)
@@ -271,21 +349,14 @@ def run_ours(args):
     attn = ps_decode.DecodeAttention.for_workload(wl, num_sms=args.sms, min_stages_per_worker=args.min_stages)
     out = torch.empty_like(wl.q)
     stream = torch.cuda.current_stream(dev)
-    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
-    flush_buf = torch.empty(max(2 * l2, 64 << 20) // 4, dtype=torch.int32, device=dev)
+    flush_buf = torch.empty(flush_bytes(dev) // 4, dtype=torch.int32, device=dev)
     flush_sink = torch.empty((), dtype=torch.int32, device=dev)
 
-    class _Flush:
+    def flush():
         """Evict the inputs from L2 between steps, outside the timed interval."""
-        nbytes = flush_buf.numel() * 4
-
-        @staticmethod
-        def zero_():
-            flush_buf.zero_()
-            if args.flush == "write-read":
-                torch.amax(flush_buf, dim=0, out=flush_sink)
-
-    flush = _Flush
+        flush_buf.zero_()
+        if args.flush == "write-read":
+            torch.amax(flush_buf, dim=0, out=flush_sink)
 
     if args.append:
         gen = torch.Generator(device=dev)
@@ -301,7 +372,7 @@ def run_ours(args):
             attn(wl.q, wl.k_cache, wl.v_cache, wl.block_table, wl.seq_lens, out=out, scale=wl.scale, stream=stream)
 
     for _ in range(max(args.warmup, 3)):
-        flush.zero_()
+        flush()
         step()
     torch.cuda.synchronize(dev)
     assert attn.device_status() == 0, "device status flags raised during warm-up"
@@ -311,22 +382,23 @@ def run_ours(args):
     for e in ev:
         for x in e:
             x.record(stream)  # create the CUDA events before the timed region
-    visible = [x.strip() for x in os.environ.get("CUDA_VISIBLE_DEVICES", "").split(",") if x.strip()]
-    gpu_index = visible[local_rank] if local_rank < len(visible) else str(local_rank)
     n_launch0 = ps_decode.ps_decode_launch_count()
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize(dev)
-    with ClockSampler(gpu_index) as clk:
+    with ClockSampler(gpu_index_of(local_rank)) as clk:
+        clk.mark_start()
         for k in range(K):
-            flush.zero_()
+            flush()
             ps_decode.ps_decode_plan_set_timing_events(attn.plan, *ev[k])
             step()
         torch.cuda.synchronize(dev)
+        clk.mark_end()
     if world > 1:
         dist.barrier()
     launches = ps_decode.ps_decode_launch_count() - n_launch0
     ps_decode.ps_decode_plan_set_timing_events(attn.plan, None, None)
+    assert attn.device_status() == 0, "device status flags raised during the timed steps"
     step_ms = [e[0].elapsed_time(e[1]) for e in ev]
     total_ms = slowest_rank_ms(sum(step_ms), dev)
 
@@ -385,51 +457,29 @@ def run_ours(args):
     # Whole job: every rank's bytes over the slowest rank's loop.
     e2e_total_ms = slowest_rank_ms(e2e_ms * e2e_steps, dev)
     e2e_value = job_throughput(alg["kv"], e2e_steps, world, e2e_total_ms)
-
-    if rank != 0:
-        if world > 1:
-            dist.barrier()
-        return None
+    info = attn.info()
+    attn.close()
+    del packs, outs, outs_h, flush_buf
 
     hbm_peak, peak_kind = measured_peaks()
     ms_per_step = total_ms / K
     value = job_throughput(alg["kv"], K, world, total_ms)
     achieved = alg["total"] / (ms_per_step * 1e-3) / 1e9
-    line = {
-        "metric": METRIC,
+    layers = MODEL_LAYERS.get(key)
+    fields = {
         "value": round(value, 2),
-        "unit": "GB/s",
-        "n_gpus": world,
-        "steps": K,
-        "warmup": args.warmup,
         "ms_per_step": round(ms_per_step, 5),
-        "higher_is_better": True,
-        "scaling": "weak",
-        "vs_baseline": None,
-        "dtype": "bf16",
-        "data": "synthetic",
-        "config": {
-            "workload": cfg.name,
-            "num_seqs": wl.num_seqs, "num_q_heads": wl.num_q_heads, "num_kv_heads": wl.num_kv_heads,
-            "head_dim": wl.head_dim, "block_size": wl.block_size, "lengths": list(cfg.lengths),
-            "seed": cfg.seed, "total_tokens": int(lens.sum()), "kv_bytes": alg["kv"],
-            "pool_blocks": wl.num_blocks,
-            "l2": "flushed before every step, outside the timed interval: %s of a %d MB buffer" % (
-                "write then read" if args.flush == "write-read" else "write", flush.nbytes >> 20),
-            "parallelism": "replicas" if world == 1 else "dp%d (independent batches per GPU)" % world,
-            "step": "append current token K/V + attend" if args.append else "attend",
-        },
-        "frac_of_hbm_peak": round(alg["total"] / (ms_per_step * 1e-3) / 1e9 / hbm_peak, 4),
+        "config": workload_config(cfg, wl, alg, flush_bytes(dev) >> 20, world, args.append),
+        "frac_of_hbm_peak": round(achieved / hbm_peak, 4),
         "decode_tokens_per_s": round(wl.num_seqs * world * K / (total_ms * 1e-3), 1),
         # Context only: one attention call per layer, so a whole model's
         # decode step over this batch needs n_layers of them.
         "attention_only_tokens_per_s": (
-            None if MODEL_LAYERS.get(args.config) is None else
-            {"n_layers": MODEL_LAYERS[args.config],
-             "value": round(wl.num_seqs * world * K / (total_ms * 1e-3) / MODEL_LAYERS[args.config], 1)}),
+            None if layers is None else
+            {"n_layers": layers, "value": round(wl.num_seqs * world * K / (total_ms * 1e-3) / layers, 1)}),
         "kernel_ms": {"mean": round(ms_per_step, 5), "median": round(statistics.median(step_ms), 5),
                       "min": round(min(step_ms), 5), "max": round(max(step_ms), 5)},
-        "frac_of_nominal_hbm": round(alg["total"] / (ms_per_step * 1e-3) / 1e9 / NOMINAL_HBM_GBS, 4),
+        "frac_of_nominal_hbm": round(achieved / NOMINAL_HBM_GBS, 4),
         "roofline": {
             "kernel": "ps_decode_kernel",
             "bound": "hbm",
@@ -438,37 +488,99 @@ def run_ours(args):
             "peak_kind": peak_kind + " (copy bandwidth, burst)",
             "unit": "GB/s",
             "frac": round(achieved / hbm_peak, 4),
-            "traffic": profiled_traffic(),
+            "traffic": None if (args.sms or args.min_stages or args.append) else profiled_traffic(
+                decode_profile_summary(cfg.name), workload=cfg.name),
             "algorithmic_bytes_per_launch": alg["total"],
         },
         "e2e": {"value": round(e2e_value, 2), "unit": "GB/s",
-                "ms_per_step": round(e2e_total_ms / e2e_steps, 5), "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-                "steps": e2e_steps,
+                "ms_per_step": round(e2e_total_ms / e2e_steps, 5), "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h, "steps": e2e_steps,
                 "overlap": "copies of step i+1 and read-back of step i-1 overlap the call of step i "
                            "(two buffer sets, three streams); time = whole loop / steps",
                 "l2": "not flushed: each step reads the whole K/V pool, larger than L2"},
         "gpu_launches": int(launches),
         "clocks": clk.summary(),
-        "plan": attn.info(),
+        "plan": info,
     }
-    if not args.no_cpu_baseline:
-        threads = os.cpu_count() or 1
-        chosen, cap = choose_oracle_sample(wl, args.cpu_seconds, threads)
-        sub = sample_for_oracle(wl, chosen, token_cap=cap)
-        spent, kv, reps = 0.0, 0, 0
-        while reps == 0 or spent < 0.8 * args.cpu_seconds:
-            dt, b = time_oracle(sub, threads)
-            spent += dt
-            kv += b
-            reps += 1
-        line["cpu_baseline"] = {
-            "value": round(kv / spent / 1e9, 4), "unit": "GB/s", "cores": threads, "kind": "oracle",
-            "sample": "%d of %d sequences%s of this workload x %d runs, fp64 oracle, %.1f s" % (
-                len(chosen), wl.num_seqs, "" if cap is None else " (first %d tokens)" % cap, reps, spent),
-        }
-    attn.close()
+    return fields, wl, alg
+
+
+def cpu_baseline_for(wl, budget_s):
+    """The oracle, as it stands, on the host cores over a bounded sample of
+    the workload (whole sequences in a seeded order, about budget_s of CPU
+    time per run, repeated to about budget_s in total)."""
+    threads = os.cpu_count() or 1
+    chosen, cap = choose_oracle_sample(wl, budget_s, threads)
+    sub = sample_for_oracle(wl, chosen, token_cap=cap)
+    spent, kv, reps = 0.0, 0, 0
+    while reps == 0 or spent < 0.8 * budget_s:
+        dt, b = time_oracle(sub, threads)
+        spent += dt
+        kv += b
+        reps += 1
+    return {
+        "value": round(kv / spent / 1e9, 4), "unit": "GB/s", "cores": threads, "kind": "oracle",
+        "sample": "%d of %d sequences%s of this workload x %d runs, fp64 oracle, %.1f s" % (
+            len(chosen), wl.num_seqs, "" if cap is None else " (first %d tokens)" % cap, reps, spent),
+    }
+
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+
+    rank, local_rank, world = dist_env()
+    if world > 1 and not dist.is_initialized():
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    keys = (args.config,) if args.config is not None else DEFAULT_CONFIGS
+    results = {}
+    head_wl = None
+    for key in keys:
+        fields, wl, _ = measure_decode(args, key, dev, rank, local_rank, world)
+        results[key] = fields
+        if key == keys[0] and rank == 0 and not args.no_cpu_baseline:
+            results[key]["cpu_baseline"] = cpu_baseline_for(wl, args.cpu_seconds)
+        del wl
+        torch.cuda.empty_cache()
     if world > 1:
         dist.barrier()
+    if rank != 0:
+        return None
+    head = results[keys[0]]
+    line = {
+        "metric": METRIC,
+        "value": head["value"],
+        "unit": "GB/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": head["ms_per_step"],
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic",
+    }
+    line.update(head)
+    if len(keys) > 1:
+        line["per_config"] = {
+            results[k]["config"]["workload"]: {
+                "value": results[k]["value"], "unit": "GB/s", "ms_per_step": results[k]["ms_per_step"],
+                "decode_tokens_per_s": results[k]["decode_tokens_per_s"],
+                "roofline": {x: results[k]["roofline"][x] for x in ("achieved", "peak", "frac", "traffic",
+                                                                     "algorithmic_bytes_per_launch")},
+                "e2e": {x: results[k]["e2e"][x] for x in ("value", "unit", "ms_per_step", "h2d_bytes_per_step",
+                                                          "d2h_bytes_per_step")},
+                "kernel_ms": results[k]["kernel_ms"],
+                "gpu_launches": results[k]["gpu_launches"],
+                "clocks": results[k]["clocks"],
+                "config": results[k]["config"],
+            } for k in keys[1:]}
+        line["gpu_launches"] = sum(results[k]["gpu_launches"] for k in keys)
+        line["gpu_launches_note"] = "headline workload %d; all timed regions of this run: %d" % (
+            head["gpu_launches"], line["gpu_launches"])
     return line
 
 
@@ -484,7 +596,7 @@ def run_transfer(args):
 
     torch.cuda.set_device(0)
     dev = torch.device("cuda", 0)
-    cfg = inputs.CONFIGS[args.config]
+    cfg = inputs.CONFIGS[args.config if args.config is not None else HEADLINE_CONFIG]
     wl = inputs.make_workload(cfg, device=dev, poison=False)
     lens = wl.seq_lens.cpu().numpy().astype(np.int64)
     Hkv, d, bs = wl.num_kv_heads, wl.head_dim, wl.block_size
@@ -511,13 +623,15 @@ def run_transfer(args):
     K = args.steps
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
     launches0 = ps_decode.ps_decode_launch_count()
-    with ClockSampler(os.environ.get("CUDA_VISIBLE_DEVICES", "0").split(",")[0] or "0") as clk:
+    with ClockSampler(gpu_index_of(0)) as clk:
+        clk.mark_start()
         for a, b in ev:
             flush_buf.zero_(); torch.amax(flush_buf, dim=0, out=sink)
             a.record(stream)
             step()
             b.record(stream)
         torch.cuda.synchronize(dev)
+        clk.mark_end()
     launches = ps_decode.ps_decode_launch_count() - launches0
     assert int(status.item()) == 0
     ms = statistics.mean(a.elapsed_time(b) for a, b in ev)
@@ -612,13 +726,15 @@ def run_prefill(args):
     K = args.steps
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
     launches0 = ps_decode.ps_decode_launch_count()
-    with ClockSampler(os.environ.get("CUDA_VISIBLE_DEVICES", "0").split(",")[0] or "0") as clk:
+    with ClockSampler(gpu_index_of(0)) as clk:
+        clk.mark_start()
         for a, b in ev:
             flush()
             a.record(stream)
             step()
             b.record(stream)
         torch.cuda.synchronize(dev)
+        clk.mark_end()
     launches = ps_decode.ps_decode_launch_count() - launches0
     assert int(status.item()) == 0, "device status %d" % int(status.item())
     ms = statistics.mean(a.elapsed_time(b) for a, b in ev)
@@ -720,23 +836,30 @@ def packed_inputs(tensors, dev, align=256):
 def run_reference(args):
     """The oracle, as it stands, on the host cores: each step runs it over a
     bounded sample of the workload sized so that the whole run stays within
-    a few minutes."""
+    a few minutes.  Same workload, metric and config object as our arm's
+    headline."""
     import torch
 
-    from paper_2608_21719_gb300 import inputs
+    from paper_2608_21719_gb300 import inputs, roofline
 
     rank, _, world = dist_env()
     if rank != 0:
         return None
-    cfg = inputs.CONFIGS[args.config]
-    dev = "cuda" if torch.cuda.is_available() else "cpu"
-    wl = inputs.make_workload(cfg, device=dev, poison=False) if dev == "cuda" or args.config == 1 else None
-    if wl is None:
-        return {"impl": "reference", "unavailable": "workload %d needs a GPU to generate its inputs" % args.config}
+    key = args.config if args.config is not None else HEADLINE_CONFIG
+    cfg = inputs.CONFIGS[key]
+    if not torch.cuda.is_available() and key != 1:
+        return {"impl": "reference", "unavailable": "workload %d needs a GPU to generate its inputs" % key}
+    dev = torch.device("cuda", 0) if torch.cuda.is_available() else torch.device("cpu")
+    wl = inputs.make_workload(cfg, device=dev, poison=False)
+    alg = roofline.algorithmic_bytes(wl.seq_lens.cpu().numpy(), wl.num_q_heads, wl.num_kv_heads, wl.head_dim,
+                                     wl.block_size)
+    flush_mb = (flush_bytes(dev) >> 20) if dev.type == "cuda" else 0
+    config = workload_config(cfg, wl, alg, flush_mb, world, args.append)
     threads = os.cpu_count() or 1
     budget = max(0.05, 150.0 / max(1, args.steps + args.warmup))
     chosen, cap = choose_oracle_sample(wl, budget, threads)
     sub = sample_for_oracle(wl, chosen, token_cap=cap)
+    del wl
     for _ in range(args.warmup):
         time_oracle(sub, threads)
     t = 0.0
@@ -746,15 +869,14 @@ def run_reference(args):
         t += dt
         kv += b
     value = kv / t / 1e9
-    sample = "%d of %d sequences%s per step" % (len(chosen), wl.num_seqs,
+    sample = "%d of %d sequences%s per step" % (len(chosen), cfg.num_seqs,
                                                 "" if cap is None else " (first %d tokens)" % cap)
     return {
         "impl": "reference",
         "metric": METRIC, "value": round(value, 4), "unit": "GB/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(t / args.steps * 1e3, 3), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": cfg.name, "num_seqs": cfg.num_seqs, "num_q_heads": cfg.num_q_heads,
-                   "num_kv_heads": cfg.num_kv_heads, "head_dim": cfg.head_dim, "block_size": cfg.block_size},
+        "config": config,
         "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": threads, "kind": "oracle",
                          "sample": sample},
         "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
