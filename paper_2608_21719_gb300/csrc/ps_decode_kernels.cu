@@ -29,7 +29,11 @@
 // counter; the warp that completes the count merges all pieces of the
 // segment in tape order by the log-sum-exp rule
 //   o = sum_c 2^(m_c - M) acc_c / sum_c 2^(m_c - M) l_c,  M = max_c m_c,
-// and resets the counter for the next call.
+// and resets the counter for the next call.  A warp whose range ends inside
+// a segment reads the segment's counter (acquire) when it starts its last
+// tile; if every other piece is already counted, it is the segment's only
+// possible merger and merges its own piece from registers, skipping the
+// partial-state write, the fence and the atomic at the kernel's tail.
 //
 // No wait spins forever: every mbarrier wait gives up after ~2 s of
 // globaltimer, raises PS_DEVICE_TIMEOUT in the workspace status word, drains
@@ -117,12 +121,30 @@ __device__ __forceinline__ void bulk_load(uint32_t dst, const void *src, uint32_
 }
 
 // 16-byte global -> shared copy that bypasses L1 (cp.async, completed by
-// cp.async.wait_all in the issuing thread).
+// cp.async.wait_group in the issuing thread).
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void *src) {
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
 }
 
-__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+// Wait until at most N of this thread's committed cp.async groups are pending.
+template <int N>
+__device__ __forceinline__ void cp_async_wait_group() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+
+// Segment counter update with acquire-release semantics at GPU scope: it
+// publishes this warp's partial state (written before it, ordered to lane 0
+// by the warp barrier) and, for the warp that completes the count, makes
+// every other piece's state visible.
+__device__ __forceinline__ int atomic_add_acq_rel(int *p, int v) {
+    int old;
+    asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+    return old;
+}
+__device__ __forceinline__ int load_acquire(const int *p) {
+    int v;
+    asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
 
 __device__ __forceinline__ void prefetch_l2(const void *p) {
     asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
@@ -323,31 +345,78 @@ __device__ __forceinline__ void accumulate_piece(float4 &acc, float &lsum, float
 
 constexpr int kStageMlBytes = 32 * (int)kSlotMl * 4;  // (m, l) of up to 32 pieces
 
+// The merging warp's own piece, still in registers (mma fragment layout:
+// lane owns heads 2 (lane & 3) and 2 (lane & 3) + 1, dims mt 16 + lane / 4
+// (+ 8)); m and l are the piece's running max and summed weights.
+struct OwnPiece {
+    const float (&acc)[8][4];
+    float m0, m1, l0, l1;
+};
+
 template <typename SlotOf>
 __device__ void merge_pieces_staged(const DecodeParams &p, int count, SlotOf slot_of, int s, int h, int lane,
-                                    uint8_t *stage) {
+                                    uint8_t *stage, int own, const OwnPiece &mine) {
     const int g = p.group;
-    const int per = min(32, (kStageArea - kStageMlBytes) / (g * kHeadDim * 4));  // pieces per acc batch
+    const int piece_bytes = g * kHeadDim * 4;
+    const int per = min(32, (kStageArea - kStageMlBytes) / piece_bytes);  // pieces the area holds at once
+    // All pieces in one batch when they fit (one L2 round trip); otherwise
+    // batches of half the area, two in flight, so that the loads of one
+    // overlap the sums of the other.
+    const bool single = count <= per;
+    const int bsz = single ? count : max(1, per / 2);
+    const int nbatch = (count + bsz - 1) / bsz;
     const uint32_t ml_base = smem_addr(stage);
     const uint32_t acc_base = ml_base + kStageMlBytes + 16u * lane;
     const uint8_t *ml_st = stage;
     const uint8_t *acc_st = stage + kStageMlBytes + 16 * lane;
-    const int my_slot = lane < count ? (int)slot_of(lane) : 0;
-    if (lane < count) {
+    const int my_slot = (lane < count && lane != own) ? (int)slot_of(lane) : 0;
+    if (lane < count && lane != own) {
         const float *src = p.ws_ml + (size_t)my_slot * kSlotMl;
 #pragma unroll
         for (int c = 0; c < (int)kSlotMl / 4; ++c) cp_async16(ml_base + (uint32_t)(lane * kSlotMl + 4 * c) * 4, src + 4 * c);
     }
-    auto issue_batch = [&](int first, int nb) {
+    auto buf_first = [&](int b) -> int { return single ? 0 : (b & 1) * bsz; };  // piece position in the area
+    auto issue_batch = [&](int b) {
+        const int first = b * bsz, nb = min(bsz, count - first);
         for (int i = 0; i < nb; ++i) {
-            const float *src = p.ws_acc + (size_t)__shfl_sync(kFull, my_slot, first + i) * kSlotFloats + 4 * lane;
+            const int piece = first + i;
+            const int slot = __shfl_sync(kFull, my_slot, piece);
+            if (piece == own) continue;
+            const float *src = p.ws_acc + (size_t)slot * kSlotFloats + 4 * lane;
             for (int n = 0; n < g; ++n)
-                cp_async16(acc_base + (uint32_t)(i * g + n) * (kHeadDim * 4), src + n * kHeadDim);
+                cp_async16(acc_base + (uint32_t)((buf_first(b) + i) * g + n) * (kHeadDim * 4), src + n * kHeadDim);
         }
+        cp_async_commit();
     };
-    issue_batch(0, min(per, count));
-    cp_async_wait_all();
-    __syncwarp();  // (m, l) rows were copied by other lanes
+    issue_batch(0);
+    if (nbatch > 1) issue_batch(1);
+    if (own >= 0) {
+        // This warp's own piece comes from its registers (single batch only):
+        // the (m, l) row and the accumulator, as the slot in the workspace
+        // would hold them.
+        float *ml_own = reinterpret_cast<float *>(stage + own * kSlotMl * 4);
+        float *acc_own = reinterpret_cast<float *>(stage + kStageMlBytes + own * piece_bytes);
+        const int h0 = 2 * (lane & 3), h1 = h0 + 1, drow = lane >> 2;
+        if (lane < 4) {
+            if (h0 < g) { ml_own[2 * h0] = mine.m0; ml_own[2 * h0 + 1] = mine.l0; }
+            if (h1 < g) { ml_own[2 * h1] = mine.m1; ml_own[2 * h1 + 1] = mine.l1; }
+        }
+#pragma unroll
+        for (int mt = 0; mt < 8; ++mt) {
+            const int d = mt * 16 + drow;
+            if (h0 < g) {
+                acc_own[h0 * kHeadDim + d] = mine.acc[mt][0];
+                acc_own[h0 * kHeadDim + d + 8] = mine.acc[mt][2];
+            }
+            if (h1 < g) {
+                acc_own[h1 * kHeadDim + d] = mine.acc[mt][1];
+                acc_own[h1 * kHeadDim + d + 8] = mine.acc[mt][3];
+            }
+        }
+    }
+    if (nbatch > 1) cp_async_wait_group<1>();
+    else cp_async_wait_group<0>();
+    __syncwarp();  // (m, l) rows and batch 0 were copied by other lanes
 
     float M[kMaxGroup];
 #pragma unroll
@@ -370,16 +439,16 @@ __device__ void merge_pieces_staged(const DecodeParams &p, int count, SlotOf slo
         acc[n] = make_float4(0.f, 0.f, 0.f, 0.f);
         lsum[n] = 0.f;
     }
-    for (int jb = 0; jb < count; jb += per) {
-        const int nb = min(per, count - jb);
-        if (jb > 0) {
+    for (int b = 0; b < nbatch; ++b) {
+        const int first = b * bsz, nb = min(bsz, count - first);
+        if (b > 0) {
+            if (b + 1 < nbatch) cp_async_wait_group<1>();
+            else cp_async_wait_group<0>();
             __syncwarp();
-            issue_batch(jb, nb);
-            cp_async_wait_all();
         }
         for (int i = 0; i < nb; ++i) {
-            const float4 *ml = reinterpret_cast<const float4 *>(ml_st + (jb + i) * kSlotMl * 4);
-            const uint8_t *src = acc_st + (size_t)i * g * (kHeadDim * 4);
+            const float4 *ml = reinterpret_cast<const float4 *>(ml_st + (first + i) * kSlotMl * 4);
+            const uint8_t *src = acc_st + (size_t)(buf_first(b) + i) * piece_bytes;
 #pragma unroll
             for (int q4 = 0; q4 < kMaxGroup / 2; ++q4) {
                 if (2 * q4 >= g) continue;
@@ -394,6 +463,10 @@ __device__ void merge_pieces_staged(const DecodeParams &p, int count, SlotOf slo
                     }
                 }
             }
+        }
+        if (b + 2 < nbatch) {
+            __syncwarp();  // every lane has read this buffer before it is refilled
+            issue_batch(b + 2);
         }
     }
     uint16_t *o = p.out + ((size_t)s * p.num_q_heads + (size_t)h * g) * kHeadDim + 4 * lane;
@@ -481,8 +554,8 @@ __device__ void merge_pieces_direct(const DecodeParams &p, int count, SlotOf slo
 
 template <typename SlotOf>
 __device__ __forceinline__ void merge_pieces(const DecodeParams &p, int count, SlotOf slot_of, int s, int h, int lane,
-                                             uint8_t *stage) {
-    if (stage != nullptr && count <= 32) merge_pieces_staged(p, count, slot_of, s, h, lane, stage);
+                                             uint8_t *stage, const OwnPiece &mine) {
+    if (stage != nullptr && count <= 32) merge_pieces_staged(p, count, slot_of, s, h, lane, stage, -1, mine);
     else merge_pieces_direct(p, count, slot_of, s, h, lane);
 }
 
@@ -701,7 +774,13 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
 
     // Finish the consume side's current piece: write its output, or leave its
     // partial state and count its tiles, merging the segment if it was last.
-    auto finalize = [&](bool ring_idle) {
+    // `others_done` (-1: not known) is the segment's tile count as read with
+    // acquire semantics while the range's last tile was consumed: when it
+    // already holds every tile but this piece's, no other warp can complete
+    // the count, so this warp is the segment's only merger and merges its
+    // own piece straight from its registers (no partial state, fence or
+    // atomic on the critical path of the kernel's tail).
+    auto finalize = [&](bool ring_idle, int others_done) {
         float L0 = l0, L1 = l1;
 #pragma unroll
         for (int o = 4; o < 32; o <<= 1) {
@@ -728,6 +807,22 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
             }
             return;
         }
+        int *cnt = p.seg_done + (size_t)s * Hkv + h;
+        const OwnPiece mine{acc, m0, m1, L0, L1};
+        // Range r0 + i holds one piece of the segment: its first piece (slot
+        // 2r) unless the range began at an earlier tile.  Only r0 can.
+        int r0, r1, cut0;
+        if (ring_idle && others_done >= 0 && others_done + c_tiles == ns) {
+            part.merge_bounds(s, h, ns, cur_rid, cur_b, cur_e, r0, r1, cut0);
+            const int count = r1 - r0 + 1;
+            const int per = min(32, (kStageArea - kStageMlBytes) / (g * kHeadDim * 4));
+            if (count <= per) {
+                auto slot_of = [&](int i) -> size_t { return 2 * (size_t)(r0 + i) + (i == 0 ? cut0 : 0); };
+                merge_pieces_staged(p, count, slot_of, s, h, lane, wbase, cur_rid - r0, mine);
+                if (lane == 0) *cnt = 0;  // nobody else touches it in this call
+                return;
+            }
+        }
         // Cut by a range boundary: leave (m, l, acc) in the range's slot.
         const size_t slotid = 2 * (size_t)cpi.z + (cpi.w ? 0 : 1);
         float *A = p.ws_acc + slotid * kSlotFloats;
@@ -751,22 +846,20 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
         __threadfence();
         __syncwarp();
         int done = 0;
-        int *cnt = p.seg_done + (size_t)s * Hkv + h;
-        if (lane == 0) done = atomicAdd(cnt, c_tiles) + c_tiles;
+        if (lane == 0) done = atomic_add_acq_rel(cnt, c_tiles) + c_tiles;
         done = __shfl_sync(kFull, done, 0);
         if (done != ns) return;
-        // This warp completed the segment: merge its pieces in tape order.
-        __threadfence();
-        // Range r0 + i holds one piece of the segment: its first piece (slot
-        // 2r) unless the range began at an earlier tile.  Only r0 can.
-        int r0, r1, cut0;
+        // This warp completed the segment (lane 0's acquire, ordered before
+        // the other lanes' reads by the shuffle's warp barrier): merge its
+        // pieces in tape order.
         part.merge_bounds(s, h, ns, cur_rid, cur_b, cur_e, r0, r1, cut0);
+        __syncwarp();
         auto slot_of = [&](int i) -> size_t { return 2 * (size_t)(r0 + i) + (i == 0 ? cut0 : 0); };
-        merge_pieces(p, r1 - r0 + 1, slot_of, s, h, lane, ring_idle ? wbase : nullptr);
+        merge_pieces(p, r1 - r0 + 1, slot_of, s, h, lane, ring_idle ? wbase : nullptr, mine);
         if (lane == 0) *cnt = 0;
     };
 
-    int consumed = 0;
+    int consumed = 0, others_done = -1;
     refill(0);
     if (p.test_stall_ns > 0 && issued > 0 &&
         !__all_sync(kFull, mbar_wait(smem_addr(&stall_bar), 0u, (unsigned long long)p.test_stall_ns))) {
@@ -791,7 +884,7 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
         const int4 meta = wmeta[slot];
         const int st = meta.x, pord = meta.y;
         if (pord != cur_piece) {
-            if (cur_piece >= 0) finalize(false);
+            if (cur_piece >= 0) finalize(false, -1);
             cur_piece = pord;
             cpi = wpieces[pord & 3];
             const uint32_t qs = smem_addr(qslots + (pord % kQSlots) * kQSlotBytes);
@@ -813,6 +906,10 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
         const uint32_t sK = smem_addr(stage), sV = sK + kTileBytes;
         const int Ls = sL[cpi.x];
         const int ns = tiles_of(Ls);
+        if (lane == 0 && consumed + 1 == issued && !(issuing && ip < cur_e) && c_tiles + 1 != ns)
+            // The range's last tile, and its piece is cut: read how much of
+            // the segment the other warps have finished (used by finalize).
+            others_done = load_acquire(p.seg_done + (size_t)cpi.x * Hkv + cpi.y);
         if (p.k_new != nullptr && st == ns - 1) {
             // Fused append: the last token of the segment is the current one.
             // Its K and V rows come from k_new / v_new (the cache slot still
@@ -907,7 +1004,8 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
         refill(consumed);
     }
     // Every copy into the ring has landed: it can stage the final merge.
-    if (cur_piece >= 0) finalize(true);
+    others_done = __shfl_sync(kFull, others_done, 0);
+    if (cur_piece >= 0) finalize(true, others_done);
 }
 
 }  // namespace
