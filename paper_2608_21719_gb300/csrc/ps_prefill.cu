@@ -1,5 +1,5 @@
 // ps_prefill.cu -- chunked-prefill attention over the paged KV cache on the
-// 5th-generation tensor cores (tcgen05 + TMEM), sm_103a.
+// 5th-generation tensor cores (tcgen05 + TMEM), 2-SM tiles, sm_103a.
 //
 // The prefill phase (PowerSlider Sec. 2.2) attends every new prompt token
 // causally over its sequence's cache; unlike decode it is a dense
@@ -8,44 +8,50 @@
 // has L_s cached tokens whose last Q_s are the new (query) tokens; query i sits
 // at position p = L_s - Q_s + i and sees keys 0 .. p.
 //
-// Tiling.  One CTA per (query tile, KV head j, sequence s).  A query tile is
-// 128 MMA rows: 128 / g consecutive query tokens times the g query heads of
-// group j (row = token * g + head), so every K/V tile staged in shared memory
-// serves the whole group.  Keys stream in tiles of 128 through shared-memory
-// rings; every 16-key chunk of a tile comes from one (block, kv-head) page of
-// the cache, addressed through the block table: for K as two TMA boxes (its
-// 64-column halves, stored [half][key][64], the K-major layout Q K^T needs),
-// for V as one box holding both halves ([chunk][half][16][64]; V is the
-// MN-major operand of P V, whose 64-column groups may sit 2 KiB apart), which
-// halves V's copies per tile.
+// Tiling.  A query tile is 128 MMA rows: 128 / g consecutive query tokens
+// times the g query heads of KV head j (row = token * g + head), so every K/V
+// tile serves the whole group.  Two CTAs on a pair of SMs (a cluster of 2)
+// take two adjacent query tiles of one (sequence, KV head) and run the
+// contractions as one M = 256 tcgen05 MMA (cta_group::2): each CTA holds its
+// own 128 query rows and half of every K/V tile -- keys 64 r .. 64 r + 63 of
+// a 128-key K tile (K-major, stored [dim half][key][64]) and dims 64 r ..
+// 64 r + 63 of all 128 keys of a V tile (MN-major, [key][64]) -- so each SM
+// stages and reads half the K/V bytes a single-SM tile would, which is what
+// the single-SM kernel ran short of (shared-memory bandwidth shared by the
+// MMA operand reads and the TMA writes).  Keys stream through per-CTA rings
+// of 16-key page slices addressed through the block table; each CTA's copies
+// complete on the leader CTA's barriers (TMA .cta_group::2), so the leader
+// issues the MMA for both once both halves have landed.  Both query tiles of
+// a pair stream the keys the later tile needs; the earlier tile masks the
+// rest.
 //
-// Per key tile n (warp roles, 7 warps):
-//   warps 0, 6 TMA producers: Q once and K_n into a three-stage ring (warp 0),
-//              V_n into a three-stage ring (warp 6).  A K stage is released
-//              as soon as its Q K^T has run, a V stage once its P V has run.
-//   warp 1     MMA issuer (one thread): S_n = Q K_n^T into one of two TMEM
-//              score buffers (M = 128, N = 128, K = 128), then, once the
-//              softmax has written P_{n-1}, O += P_{n-1} V_{n-1} with P read
-//              from TMEM and V (MN-major) from shared memory, into the TMEM
-//              output accumulator.  Completion is signalled with
-//              tcgen05.commit on mbarriers.
-//   warps 2-5  softmax, one TMEM lane (= one row) per thread: load the score
-//              row, mask it causally, update the running max m and sum l in
-//              fp32 (base 2, log2 e folded into the scale), write the bf16
-//              probabilities into TMEM P buffer n & 1 (the A operand of the
-//              P V MMA), and rescale the output row in TMEM when the max has
-//              grown.  Only that rescale waits for the previous P V, so the
-//              exponentials of tile n+1 overlap the P V of tile n.
+// Per key tile n (warp roles, 7 warps per CTA):
+//   warp 0     TMA: Q once, then this CTA's half of K_n into a K ring.
+//   warp 6     TMA: this CTA's half of V_n into a V ring; the last tile's rows
+//              past the needed keys are zeroed (its copy completes locally
+//              first) before the leader is told.
+//   warp 1     leader CTA only, one thread: S_n = Q K_n^T into one of two TMEM
+//              score buffers of both CTAs (M = 256, N = 128, K = 128), then,
+//              once both CTAs' softmax has written P_{n-1}, O += P_{n-1}
+//              V_{n-1} with P read from TMEM; tcgen05.commit multicasts each
+//              completion to both CTAs' barriers.
+//   warps 2-5  softmax, one TMEM lane (= one row) per thread, in each CTA:
+//              load the score row, mask it causally, update the running max
+//              m and sum l in fp32 (base 2, log2 e folded into the scale),
+//              write the bf16 probabilities into TMEM P buffer n & 1 (the A
+//              operand of the P V MMA), and rescale the output row in TMEM
+//              when the max has grown.
 // The rescale is lazy: the reference max m only moves when the tile max
 // exceeds it by more than 2^8, so P <= 256 and no value leaves fp32/bf16
 // range; the final O / l is the same quotient whichever reference max was
-// used.  The QK^T of tile n+1 runs on the tensor cores while the softmax works
-// on tile n.
+// used.
 //
 // Every mbarrier wait gives up after ~2 s of globaltimer, or at once when
-// another role has given up, and raises PS_DEVICE_TIMEOUT in the optional
-// device status word; the producer then waits for its own copies, the MMA
-// issuer for its own MMAs, and TMEM is freed on every path.
+// another role of its CTA has given up, and raises PS_DEVICE_TIMEOUT in the
+// optional device status word; the producers then wait for their own copies,
+// the MMA issuer for its own MMAs, both CTAs meet at a cluster barrier, and
+// TMEM is freed on every path.
+
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -60,29 +66,34 @@
 namespace {
 
 constexpr int kD = 128;            // head_dim
-constexpr int kRows = 128;         // MMA M: query rows per tile
+constexpr int kRows = 128;         // query rows per CTA (MMA M = 256 over the pair)
 constexpr int kKeys = 128;         // MMA N of S, K of P.V: keys per tile
 constexpr int kChunk = 16;         // keys per TMA box (one page slice)
 #ifndef PS_PREFILL_KSTAGES
-#define PS_PREFILL_KSTAGES 3
+#define PS_PREFILL_KSTAGES 5
 #endif
 #ifndef PS_PREFILL_VSTAGES
-#define PS_PREFILL_VSTAGES 3
+#define PS_PREFILL_VSTAGES 5
 #endif
 constexpr int kKStages = PS_PREFILL_KSTAGES;  // K ring: a stage is free once its Q K^T is done
 constexpr int kVStages = PS_PREFILL_VSTAGES;  // V ring: a stage is free once its P V is done
 constexpr int kThreads = 224;
-constexpr int kHalf = kRows * 64 * 2;   // one 64-column half of a 128-row tile: 16 KiB
-constexpr int kTile = 2 * kHalf;        // 32 KiB
+constexpr int kHalfQ = kRows * 64 * 2;        // one 64-column half of the 128-row Q tile: 16 KiB
+constexpr int kQBytes = 2 * kHalfQ;           // 32 KiB
+constexpr int kPairKeys = kKeys / 2;          // keys of each K tile one CTA holds
+constexpr int kKHalf = kPairKeys * 128;       // one 64-dim half of a CTA's K slice: 8 KiB
+constexpr int kKStage = 2 * kKHalf;           // 16 KiB
+constexpr int kVStage = kKeys * 128;          // 128 keys x this CTA's 64 dims: 16 KiB
 constexpr int kOffQ = 0;
-constexpr int kOffK = kOffQ + kTile;
-constexpr int kOffV = kOffK + kKStages * kTile;
-constexpr int kOffBar = kOffV + kVStages * kTile;
-constexpr int kSmemBytes = 1024 + kOffBar + 256;  // 1 KiB of alignment slack
+constexpr int kOffK = kOffQ + kQBytes;
+constexpr int kOffV = kOffK + kKStages * kKStage;
+constexpr int kOffBar = kOffV + kVStages * kVStage;
+constexpr int kBarBytes = 512;
+constexpr int kSmemBytes = 1024 + kOffBar + kBarBytes;  // 1 KiB of alignment slack
 static_assert(kSmemBytes <= 227 * 1024, "shared memory");
 constexpr uint32_t kTmemCols = 512;
-// TMEM columns: S buffers at 0 and 128, O at 256, two P buffers (bf16 pairs
-// packed in 32-bit columns, 64 columns each) at 384 and 448.
+// TMEM columns (the same in both CTAs): S buffers at 0 and 128, O at 256, two
+// P buffers (bf16 pairs packed in 32-bit columns, 64 columns each) at 384 and 448.
 constexpr uint32_t kColO = 256, kColP = 384;
 constexpr float kRescaleLog2 = 8.0f;
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;
@@ -108,9 +119,6 @@ __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
 __device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
 }
-__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
 __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
     uint32_t ok;
     asm volatile(
@@ -130,22 +138,6 @@ __device__ __forceinline__ unsigned long long global_ns() {
 __device__ __forceinline__ void fence_proxy_async_smem() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
-__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *tm, int c0, int c1, int c2,
-                                            uint32_t bar) {
-    asm volatile(
-        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-        " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
-        "l"(reinterpret_cast<uint64_t>(tm)), "r"(c0), "r"(c1), "r"(c2), "r"(bar)
-        : "memory");
-}
-// The same with an L2 cache-policy hint (from createpolicy).
-__device__ __forceinline__ void tma_load_4d_hint(uint32_t dst, const CUtensorMap *tm, int c0, int c1, int c2, int c3,
-                                                 uint32_t bar, uint64_t policy) {
-    asm volatile("cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
-        " [%0], [%1, {%2, %3, %4, %5}], [%6], %7;" ::"r"(dst), "l"(reinterpret_cast<uint64_t>(tm)), "r"(c0), "r"(c1),
-        "r"(c2), "r"(c3), "r"(bar), "l"(policy) : "memory");
-}
-
 __device__ __forceinline__ void tma_load_3d_hint(uint32_t dst, const CUtensorMap *tm, int c0, int c1, int c2,
                                                  uint32_t bar, uint64_t policy) {
     asm volatile(
@@ -172,25 +164,68 @@ __host__ __device__ constexpr uint32_t instr_desc(int m, int n, int b_mn) {
     return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)b_mn << 16) | ((uint32_t)(n >> 3) << 17) |
            ((uint32_t)(m >> 4) << 24);
 }
-__device__ __forceinline__ void umma(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+// D (both CTAs' TMEM) += A . B over the CTA pair: each CTA supplies its 128
+// rows of A and its half (along N) of B at the same shared-memory offsets.
+__device__ __forceinline__ void umma2(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
     asm volatile(
         "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
         "l"(a), "l"(b), "r"(idesc), "r"(acc)
         : "memory");
 }
-// The same with A read from tensor memory (row = TMEM lane, K packed in bf16
-// pairs along the columns: a K step of 16 is 8 columns).
-__device__ __forceinline__ void umma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b, uint32_t idesc, uint32_t acc) {
+// The same with A read from each CTA's tensor memory (row = TMEM lane, K
+// packed in bf16 pairs along the columns: a K step of 16 is 8 columns).
+__device__ __forceinline__ void umma2_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b, uint32_t idesc, uint32_t acc) {
     asm volatile(
         "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
         "r"(a_tmem), "l"(b), "r"(idesc), "r"(acc)
         : "memory");
 }
-__device__ __forceinline__ void umma_commit(uint32_t bar) {
-    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+// Arrive on the barrier at this offset in both CTAs of the pair once every
+// MMA issued so far has completed.
+__device__ __forceinline__ void umma_commit_pair(uint32_t bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(bar),
+        "h"((uint16_t)3)
+        : "memory");
+}
+__device__ __forceinline__ uint32_t cta_rank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+// Shared::cluster address of the same shared-memory location in CTA `rank`.
+__device__ __forceinline__ uint32_t map_to(uint32_t addr, uint32_t rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+    return r;
+}
+// Arrive on a barrier of either CTA of the pair.  The arrivals carry the
+// default (CTA-scope release) semantics: what they order -- tensor-memory
+// reads and writes finished with tcgen05.wait and fenced with
+// tcgen05.fence::before_thread_sync, and TMA transfers counted by the
+// barrier itself -- needs no cluster-scope release, which costs ~1-2 us of
+// latency per arrival on this path.
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_bar) {
+    asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(cluster_bar) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx_cluster(uint32_t cluster_bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cluster.b64 _, [%0], %1;" ::"r"(cluster_bar), "r"(bytes)
                  : "memory");
+}
+__device__ __forceinline__ void cluster_sync() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// TMA load into this CTA's shared memory whose completion is counted on a
+// barrier of either CTA of the pair (`cluster_bar`), with an L2 policy.
+__device__ __forceinline__ void tma_load_3d_pair(uint32_t dst, const CUtensorMap *tm, int c0, int c1, int c2,
+                                                 uint32_t cluster_bar, uint64_t policy) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.cta_group::2.L2::cache_hint"
+        " [%0], [%1, {%2, %3, %4}], [%5], %6;" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(tm)), "r"(c0), "r"(c1), "r"(c2), "r"(cluster_bar), "l"(policy)
+        : "memory");
 }
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float *v) {
     uint32_t r[32];
@@ -275,80 +310,87 @@ __device__ __forceinline__ void drain_phase(uint32_t bar, uint32_t parity) {
 }
 
 
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     ps_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                       const __grid_constant__ CUtensorMap tmV, const PrefillParams p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    // Consecutive CTAs share a (sequence, KV head), heaviest (last) query
-    // tile first: the few K/V streams in flight at a time stay in L2.
-    const int qt = p.num_qtiles - 1 - (int)blockIdx.x;
+    const uint32_t rank = cta_rank();  // 0: the leader, which issues the MMAs
+    // Consecutive pairs share a (sequence, KV head), heaviest (last) query
+    // tiles first: the few K/V streams in flight at a time stay in L2.  The
+    // leader takes the later tile of its pair, the other CTA the one before
+    // (which may not exist: tile -1).
+    const int qt_hi = p.num_qtiles - 1 - 2 * (int)(blockIdx.x >> 1);
+    const int qt = qt_hi - (int)rank;
     const int j = blockIdx.y, s = blockIdx.z;
     const int g = p.group, tpt = p.tokens_per_tile;
 
-    // Sequence geometry (uniform over the CTA).
+    // Sequence geometry (uniform over the pair).
     const int qs0 = __ldg(p.q_start + s), qs1 = __ldg(p.q_start + s + 1);
     const int Q = qs1 - qs0;
     const int L = __ldg(p.seq_lens + s);
-    const int tok0 = qt * tpt;
     // max_q_len below a chunk leaves that chunk's later rows uncovered.
-    if (qt == p.num_qtiles - 1 && j == 0 && tid == 0 && Q > p.num_qtiles * tpt && p.status)
+    if (qt_hi == p.num_qtiles - 1 && rank == 0 && j == 0 && tid == 0 && Q > p.num_qtiles * tpt && p.status)
         atomicOr(p.status, (unsigned)PS_DEVICE_LEN_CLAMPED);
-    if (tok0 >= Q) return;
+    if (max(qt_hi - 1, 0) * tpt >= Q) return;  // neither tile of the pair has rows
     const long long cap = (long long)p.max_blocks_per_seq * p.block_size;
     if (Q < 0 || L < Q || (long long)L > cap || qs0 < 0 || qs1 > p.total_q) {
-        if (tid == 0 && j == 0 && p.status) atomicOr(p.status, (unsigned)PS_DEVICE_LEN_CLAMPED);
+        if (tid == 0 && rank == 0 && j == 0 && p.status) atomicOr(p.status, (unsigned)PS_DEVICE_LEN_CLAMPED);
         return;
     }
-    const int tok_end = min(Q, tok0 + tpt);
-    const int kv_limit = L - Q + tok_end;  // keys this tile needs: [0, kv_limit)
+    const int tok0 = qt * tpt;                       // negative for the missing tile -1
+    const int kv_limit = L - Q + min(Q, (qt_hi + 1) * tpt);  // keys the pair needs: [0, kv_limit)
     const int ntiles = (kv_limit + kKeys - 1) / kKeys;
 
     uint64_t *bars = reinterpret_cast<uint64_t *>(sm + kOffBar);
     const uint32_t bar_q = saddr(bars + 0);
-    auto bar_kfull = [&](int st) { return saddr(bars + 1 + st); };                        // [kKStages]
-    auto bar_kfree = [&](int st) { return saddr(bars + 1 + kKStages + st); };             // [kKStages]
-    auto bar_vfull = [&](int st) { return saddr(bars + 1 + 2 * kKStages + st); };         // [kVStages]
+    auto bar_kfull = [&](int st) { return saddr(bars + 1 + st); };                         // [kKStages], leader's
+    auto bar_kfree = [&](int st) { return saddr(bars + 1 + kKStages + st); };              // [kKStages]
+    auto bar_vfull = [&](int st) { return saddr(bars + 1 + 2 * kKStages + st); };          // [kVStages], leader's
     auto bar_vfree = [&](int st) { return saddr(bars + 1 + 2 * kKStages + kVStages + st); };
     constexpr int kB = 1 + 2 * kKStages + 2 * kVStages;
     auto bar_sfull = [&](int b) { return saddr(bars + kB + b); };
-    auto bar_sfree = [&](int b) { return saddr(bars + kB + 2 + b); };
-    auto bar_pfull = [&](int b) { return saddr(bars + kB + 4 + b); };
+    auto bar_sfree = [&](int b) { return saddr(bars + kB + 2 + b); };  // leader's
+    auto bar_pfull = [&](int b) { return saddr(bars + kB + 4 + b); };  // leader's
     auto bar_pfree = [&](int b) { return saddr(bars + kB + 6 + b); };
     const uint32_t bar_mma_end = saddr(bars + kB + 8);
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + kB + 9);
-    volatile int *abort = reinterpret_cast<volatile int *>(bars + kB + 10);
-    static_assert((1 + 2 * kKStages + 2 * kVStages + 11) * 8 <= 256, "barrier area");
+    const uint32_t bar_vtail = saddr(bars + kB + 9);
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + kB + 10);
+    volatile int *abort = reinterpret_cast<volatile int *>(bars + kB + 11);
+    static_assert((1 + 2 * kKStages + 2 * kVStages + 12) * 8 <= kBarBytes, "barrier area");
 
     if (tid == 0) {
-        mbar_init(bar_q, 1);
+        mbar_init(bar_q, 2);  // one arrival (with its bytes) from each CTA
         for (int i = 0; i < kKStages; ++i) {
-            mbar_init(bar_kfull(i), 1);
+            mbar_init(bar_kfull(i), 2);
             mbar_init(bar_kfree(i), 1);
         }
         for (int i = 0; i < kVStages; ++i) {
-            mbar_init(bar_vfull(i), 1);
+            mbar_init(bar_vfull(i), 2);
             mbar_init(bar_vfree(i), 1);
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(bar_sfull(i), 1);
-            mbar_init(bar_sfree(i), 4);
-            mbar_init(bar_pfull(i), 128);
+            mbar_init(bar_sfree(i), 8);  // four softmax warps in each CTA
+            mbar_init(bar_pfull(i), 8);
             mbar_init(bar_pfree(i), 1);
         }
         mbar_init(bar_mma_end, 1);
+        mbar_init(bar_vtail, 1);
         *abort = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     if (warp == 1) {
-        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(saddr(tmem_slot)),
+        asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(saddr(tmem_slot)),
                      "r"(kTmemCols)
                      : "memory");
-        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
     }
+    // Both CTAs' barriers exist and their TMEM is allocated before either
+    // CTA's copies or arrivals can reach the other.
     tc_fence_before();
-    __syncthreads();
+    cluster_sync();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
@@ -357,116 +399,145 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp == 0 || warp == 6) {
         // ----------------------------------------------------- producers --
         const bool is_k = warp == 0;
+        uint64_t keep;  // every K/V page is read by all query tiles of its (sequence, head)
+        asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(keep));
         if (is_k && lane == 0) {
             asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmQ)) : "memory");
             asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
-            mbar_expect_tx(bar_q, (uint32_t)(2 * 128 * g * tpt));
-            tma_load_3d(sQ, &tmQ, 0, j * g, qs0 + tok0, bar_q);
-            tma_load_3d(sQ + kHalf, &tmQ, 64, j * g, qs0 + tok0, bar_q);
+            const uint32_t lq = map_to(bar_q, 0);
+            mbar_expect_tx_cluster(lq, (uint32_t)(2 * 128 * g * tpt));
+            // Rows of a missing or empty tile read zeros or other rows; they are never written.
+            tma_load_3d_pair(sQ, &tmQ, 0, j * g, qs0 + tok0, lq, keep);
+            tma_load_3d_pair(sQ + kHalfQ, &tmQ, 64, j * g, qs0 + tok0, lq, keep);
         }
         if (!is_k && lane == 0)
             asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
         const int stages = is_k ? kKStages : kVStages;
-        const uint32_t ring = is_k ? sK : sV;
-        const CUtensorMap *tm = is_k ? &tmK : &tmV;
         const int *bt_row = p.block_table + (size_t)s * p.max_blocks_per_seq;
-        const int half = (lane >> 3) & 1, c = lane & 7;  // K: lanes 0-15, 8 chunks x 2 halves; V: lanes 0-7
-        // Every K/V page is read by all query tiles of its (sequence, head):
-        // ask L2 to keep it (evict last).
-        uint64_t keep;
-        asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(keep));
         int issued = 0;
+        bool tail_done = false;
         for (int n = 0; n < ntiles; ++n) {
             const int st = n % stages, use = n / stages;
-            if (n >= stages &&
-                !warp_wait(is_k ? bar_kfree(st) : bar_vfree(st), (use - 1) & 1, abort, p.status))
+            if (n >= stages && !warp_wait(is_k ? bar_kfree(st) : bar_vfree(st), (use - 1) & 1, abort, p.status))
                 break;
             const int base = n * kKeys;
-            const int nc = (min(kKeys, kv_limit - base) + kChunk - 1) / kChunk;
-            const uint32_t full = is_k ? bar_kfull(st) : bar_vfull(st);
-            if (lane == 0) mbar_expect_tx(full, (uint32_t)(nc * 2 * kChunk * 128));
-            __syncwarp();
-            if (is_k ? (lane < 16 && c < nc) : (lane < nc)) {
-                const int cc = is_k ? c : lane;
-                const int t0 = base + cc * kChunk;
-                const int lb = t0 / p.block_size;
-                const int b = __ldg(bt_row + lb);
-                int page = -1;  // out of range: TMA fills zeros
-                if (b >= 0 && (long long)b < p.num_blocks) page = b * p.num_kv_heads + j;
-                else if (p.status && is_k) atomicOr(p.status, (unsigned)PS_DEVICE_BAD_BLOCK);
-                if (is_k)
-                    tma_load_3d_hint(ring + st * kTile + half * kHalf + cc * (kChunk * 128), tm, half * 64,
+            if (is_k) {
+                // Keys 64 rank .. 64 rank + 63 of the tile, both 64-dim halves:
+                // lanes 0-7 take (chunk lane & 3, half lane >> 2).
+                const int k0 = base + kPairKeys * (int)rank;
+                const int nc = max(0, min(kPairKeys / kChunk, (kv_limit - k0 + kChunk - 1) / kChunk));
+                const uint32_t full = map_to(bar_kfull(st), 0);
+                if (lane == 0) mbar_expect_tx_cluster(full, (uint32_t)(nc * 2 * kChunk * 128));
+                __syncwarp();
+                const int c = lane & 3, half = lane >> 2;
+                if (lane < 8 && c < nc) {
+                    const int t0 = k0 + c * kChunk;
+                    const int lb = t0 / p.block_size;
+                    const int b = __ldg(bt_row + lb);
+                    int page = -1;  // out of range: TMA fills zeros
+                    if (b >= 0 && (long long)b < p.num_blocks) page = b * p.num_kv_heads + j;
+                    else if (p.status) atomicOr(p.status, (unsigned)PS_DEVICE_BAD_BLOCK);
+                    tma_load_3d_pair(sK + st * kKStage + half * kKHalf + c * (kChunk * 128), &tmK, half * 64,
                                      t0 - lb * p.block_size, page, full, keep);
-                else  // both 64-column halves of the chunk in one box: [half][16][64]
-                    tma_load_4d_hint(ring + st * kTile + cc * (2 * kChunk * 128), tm, 0, t0 - lb * p.block_size, 0,
-                                     page, full, keep);
+                }
+            } else {
+                // Dims 64 rank .. 64 rank + 63 of all keys of the tile: lane c takes chunk c.
+                const int valid = min(kKeys, kv_limit - base);
+                const int nc = (valid + kChunk - 1) / kChunk;
+                const bool tail = valid < kKeys;
+                const uint32_t full = map_to(bar_vfull(st), 0);
+                if (lane == 0) {
+                    if (tail) mbar_expect_tx(bar_vtail, (uint32_t)(nc * kChunk * 128));
+                    else mbar_expect_tx_cluster(full, (uint32_t)(nc * kChunk * 128));
+                }
+                __syncwarp();
+                if (lane < nc) {
+                    const int t0 = base + lane * kChunk;
+                    const int lb = t0 / p.block_size;
+                    const int b = __ldg(bt_row + lb);
+                    int page = -1;
+                    if (b >= 0 && (long long)b < p.num_blocks) page = b * p.num_kv_heads + j;
+                    const uint32_t dst = sV + st * kVStage + lane * (kChunk * 128);
+                    if (tail) tma_load_3d_hint(dst, &tmV, 64 * (int)rank, t0 - lb * p.block_size, page, bar_vtail, keep);
+                    else tma_load_3d_pair(dst, &tmV, 64 * (int)rank, t0 - lb * p.block_size, page, full, keep);
+                }
+                issued = n + 1;
+                if (tail) {
+                    // The last tile: its copy completes here first, then the rows
+                    // past the needed keys (other tokens' data, or stale bytes)
+                    // are zeroed -- P is zero there -- before the leader is told.
+                    if (!warp_wait(bar_vtail, 0, abort, p.status)) break;
+                    tail_done = true;
+                    uint8_t *v = sm + kOffV + st * kVStage;
+                    for (int e = lane; e < (kKeys - valid) * 8; e += 32)
+                        *reinterpret_cast<uint4 *>(v + (valid + (e >> 3)) * 128 + (e & 7) * 16) = make_uint4(0, 0, 0, 0);
+                    fence_proxy_async_smem();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive_cluster(full);
+                }
             }
             issued = n + 1;
         }
-        // Drain: the last copies of each stage must land before the CTA exits.
-        for (int n = max(0, issued - stages); n < issued; ++n)
-            drain_phase(is_k ? bar_kfull(n % stages) : bar_vfull(n % stages), (n / stages) & 1);
-        if (is_k) drain_phase(bar_q, 0);
+        // Drain: this CTA's copies must land before it can leave.  Copies that
+        // count on the leader's barriers are covered by the leader's waits and
+        // the final cluster barrier; the local ones are waited for here.
+        if (!is_k && !tail_done && issued > 0 && min(kKeys, kv_limit - (issued - 1) * kKeys) < kKeys)
+            drain_phase(bar_vtail, 0);
+        if (rank == 0) {
+            for (int n = max(0, issued - stages); n < issued; ++n)
+                drain_phase(is_k ? bar_kfull(n % stages) : bar_vfull(n % stages), (n / stages) & 1);
+            if (is_k) drain_phase(bar_q, 0);
+        }
     } else if (warp == 1) {
-        // ---------------------------------------------------- MMA issuer --
-        constexpr uint32_t idS = instr_desc(kRows, kKeys, 0);
-        constexpr uint32_t idO = instr_desc(kRows, kD, 1);
-        bool ok = warp_wait(bar_q, 0, abort, p.status);
-        for (int n = 0; ok && n <= ntiles; ++n) {
-            if (n < ntiles) {
-                const int st = n % kKStages, b = n & 1;
-                if (!warp_wait(bar_kfull(st), (n / kKStages) & 1, abort, p.status)) { ok = false; break; }
-                if (n >= 2 && !warp_wait(bar_sfree(b), ((n >> 1) - 1) & 1, abort, p.status)) { ok = false; break; }
-                tc_fence_after();
-                if (lane == 0) {
-                    const uint32_t kb = sK + st * kTile;
+        if (rank == 0) {
+            // ---------------------------------------- MMA issuer (leader) --
+            constexpr uint32_t idS = instr_desc(2 * kRows, kKeys, 0);
+            constexpr uint32_t idO = instr_desc(2 * kRows, kD, 1);
+            bool ok = warp_wait(bar_q, 0, abort, p.status);
+            // Descriptor bases, once: a stage or K-step offset is an add to the
+            // 14-bit start-address field (shared-memory addresses stay below 256 KiB).
+            const uint64_t dQ = smem_desc(sQ, 16, 1024), dK = smem_desc(sK, 16, 1024), dV = smem_desc(sV, 16, 1024);
+            for (int n = 0; ok && n <= ntiles; ++n) {
+                if (n < ntiles) {
+                    const int st = n % kKStages, b = n & 1;
+                    if (!warp_wait(bar_kfull(st), (n / kKStages) & 1, abort, p.status)) { ok = false; break; }
+                    if (n >= 2 && !warp_wait(bar_sfree(b), ((n >> 1) - 1) & 1, abort, p.status)) { ok = false; break; }
+                    tc_fence_after();
+                    if (lane == 0) {
+                        const uint64_t kd = dK + (uint64_t)((st * kKStage) >> 4);
 #pragma unroll
-                    for (int kk = 0; kk < kD / 16; ++kk) {
-                        const uint32_t off = (kk >> 2) * kHalf + (kk & 3) * 32;
-                        umma(tmem + b * kKeys, smem_desc(sQ + off, 16, 1024), smem_desc(kb + off, 16, 1024), idS,
-                             kk > 0);
+                        for (int kk = 0; kk < kD / 16; ++kk) {
+                            umma2(tmem + b * kKeys, dQ + (uint64_t)(((kk >> 2) * kHalfQ + (kk & 3) * 32) >> 4),
+                                  kd + (uint64_t)(((kk >> 2) * kKHalf + (kk & 3) * 32) >> 4), idS, kk > 0);
+                        }
+                        umma_commit_pair(bar_sfull(b));
+                        umma_commit_pair(bar_kfree(st));
                     }
-                    umma_commit(bar_sfull(b));
-                    umma_commit(bar_kfree(st));
-                }
-                __syncwarp();
-            }
-            if (n >= 1) {
-                const int m = n - 1, st = m % kVStages;
-                if (!warp_wait(bar_vfull(st), (m / kVStages) & 1, abort, p.status)) { ok = false; break; }
-                const uint32_t vb = sV + st * kTile;
-                const int valid = kv_limit - m * kKeys;
-                if (valid < kKeys) {
-                    // Rows past the last needed key hold other tokens' data
-                    // or stale bytes; P is zero there, so make V zero too.
-                    uint8_t *v = sm + kOffV + st * kTile;
-                    const int nvec = (kKeys - valid) * 8;
-                    for (int e = lane; e < 2 * nvec; e += 32) {
-                        const int h = e / nvec, r = e - h * nvec;
-                        const int key = valid + (r >> 3);
-                        *reinterpret_cast<uint4 *>(v + (key >> 4) * (2 * kChunk * 128) + h * (kChunk * 128) +
-                                                   (key & 15) * 128 + (r & 7) * 16) = make_uint4(0, 0, 0, 0);
-                    }
-                    fence_proxy_async_smem();
                     __syncwarp();
                 }
-                if (!warp_wait(bar_pfull(m & 1), (m >> 1) & 1, abort, p.status)) { ok = false; break; }
-                tc_fence_after();
-                if (lane == 0) {
-                    const uint32_t pt = tmem + kColP + (m & 1) * (kKeys / 2);
+                if (n >= 1) {
+                    const int m = n - 1, st = m % kVStages;
+                    if (!warp_wait(bar_vfull(st), (m / kVStages) & 1, abort, p.status)) { ok = false; break; }
+                    if (!warp_wait(bar_pfull(m & 1), (m >> 1) & 1, abort, p.status)) { ok = false; break; }
+                    tc_fence_after();
+                    if (lane == 0) {
+                        const uint32_t pt = tmem + kColP + (m & 1) * (kKeys / 2);
+                        const uint64_t vd = dV + (uint64_t)((st * kVStage) >> 4);
 #pragma unroll
-                    for (int kk = 0; kk < kKeys / 16; ++kk)
-                        umma_ts(tmem + kColO, pt + kk * 8, smem_desc(vb + kk * 4096, 2048, 1024), idO,
-                                (m > 0 || kk > 0) ? 1u : 0u);
-                    umma_commit(bar_pfree(m & 1));
-                    umma_commit(bar_vfree(st));
+                        for (int kk = 0; kk < kKeys / 16; ++kk)
+                            umma2_ts(tmem + kColO, pt + kk * 8, vd + (uint64_t)((kk * (16 * 128)) >> 4), idO,
+                                     (m > 0 || kk > 0) ? 1u : 0u);
+                        umma_commit_pair(bar_pfree(m & 1));
+                        umma_commit_pair(bar_vfree(st));
+                    }
+                    __syncwarp();
                 }
-                __syncwarp();
             }
+            // Every MMA issued above has finished, in both CTAs, before TMEM
+            // and shared memory go away.
+            if (lane == 0) umma_commit_pair(bar_mma_end);
+            __syncwarp();
         }
-        // Every MMA issued above has finished before TMEM and smem go away.
-        if (lane == 0) umma_commit(bar_mma_end);
-        __syncwarp();
         drain_phase(bar_mma_end, 0);
     } else {
         // ------------------------------------------------------- softmax --
@@ -474,7 +545,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int r = quarter * 32 + lane;
         const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
         const int tl = r / g, hl = r - tl * g;
-        const bool row_valid = (tl < tpt) && (tok0 + tl < Q);
+        const bool row_valid = (tl < tpt) && (qt >= 0) && (tok0 + tl < Q);
         const int limit = row_valid ? (L - Q + tok0 + tl + 1) : kv_limit;
         const float sl2 = p.scale_log2;
         float m_ref = -INFINITY, l = 0.f;
@@ -490,7 +561,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             tmem_loaded<kKeys>(sv);
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(bar_sfree(b));
+            if (lane == 0) mbar_arrive_cluster(map_to(bar_sfree(b), 0));
             const int base = n * kKeys;
             if (base + kKeys > limit) {
 #pragma unroll
@@ -546,7 +617,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             tmem_wait_st();
             tc_fence_before();
-            mbar_arrive(bar_pfull(b));
+            __syncwarp();
+            if (lane == 0) mbar_arrive_cluster(map_to(bar_pfull(b), 0));
         }
         if (ok && warp_wait(bar_pfree((ntiles - 1) & 1), ((ntiles - 1) >> 1) & 1, abort, p.status)) {
             tc_fence_after();
@@ -573,11 +645,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
         }
     }
+    // Neither CTA leaves (nor frees TMEM) while the other may still touch its
+    // shared memory or the leader's MMAs may still run.
     tc_fence_before();
     __syncthreads();
+    cluster_sync();
     if (warp == 1) {
         tc_fence_after();
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
+        asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
     }
 }
 
@@ -609,21 +684,6 @@ bool encode3d(CUtensorMap *tm, const void *base, cuuint64_t d1, cuuint64_t d2, c
     cuuint32_t box[3] = {64, b1, b2};
     cuuint32_t estr[3] = {1, 1, 1};
     return fn(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims, strides, box, estr,
-              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
-// V as [page][slot][half][64]: dims (64, slot, half, page) with the half
-// stride (128 B) inside the slot stride (256 B), so that one box {64, 16, 2}
-// lands as [half][16][64] (both halves of a 16-key chunk in one copy).
-bool encode_v4d(CUtensorMap *tm, const void *base, cuuint64_t bs, cuuint64_t pages) {
-    EncodeTiledFn fn = encoder();
-    if (!fn) return false;
-    cuuint64_t dims[4] = {64, bs, 2, pages};
-    cuuint64_t strides[3] = {(cuuint64_t)kD * 2, 64 * 2, bs * kD * 2};
-    cuuint32_t box[4] = {64, kChunk, 2, 1};
-    cuuint32_t estr[4] = {1, 1, 1, 1};
-    return fn(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(base), dims, strides, box, estr,
               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
@@ -660,7 +720,7 @@ extern "C" ps_status_t ps_prefill_attention(const void *q, const void *k_cache, 
     CUtensorMap tmQ, tmK, tmV;
     if (!encode3d(&tmQ, q, (cuuint64_t)num_q_heads, (cuuint64_t)total_q_tokens, (cuuint32_t)g, (cuuint32_t)tpt) ||
         !encode3d(&tmK, k_cache, (cuuint64_t)block_size, (cuuint64_t)(num_blocks * num_kv_heads), kChunk, 1) ||
-        !encode_v4d(&tmV, v_cache, (cuuint64_t)block_size, (cuuint64_t)(num_blocks * num_kv_heads)))
+        !encode3d(&tmV, v_cache, (cuuint64_t)block_size, (cuuint64_t)(num_blocks * num_kv_heads), kChunk, 1))
         return PS_ERR_CUDA;
     // The shared-memory limit is a per-device function attribute: set it for
     // the current device on every call (cheap), so that a process driving
@@ -686,7 +746,8 @@ extern "C" ps_status_t ps_prefill_attention(const void *q, const void *k_cache, 
     pp.max_blocks_per_seq = max_blocks_per_seq;
     pp.num_blocks = num_blocks;
     pp.scale_log2 = scale * 1.4426950408889634f;
-    const dim3 grid((unsigned)nqt, (unsigned)num_kv_heads, (unsigned)num_seqs);
+    // Clusters of two CTAs, one pair per two adjacent query tiles.
+    const dim3 grid((unsigned)(2 * ((nqt + 1) / 2)), (unsigned)num_kv_heads, (unsigned)num_seqs);
     if (ps::take_injected_launch_error() != cudaSuccess) return PS_ERR_CUDA;
     ps_prefill_kernel<<<grid, kThreads, kSmemBytes, reinterpret_cast<cudaStream_t>(stream)>>>(tmQ, tmK, tmV, pp);
     if (cudaGetLastError() != cudaSuccess) return PS_ERR_CUDA;
