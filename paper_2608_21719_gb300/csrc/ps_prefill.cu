@@ -40,7 +40,13 @@
 //              m and sum l in fp32 (base 2, log2 e folded into the scale),
 //              write the bf16 probabilities into TMEM P buffer n & 1 (the A
 //              operand of the P V MMA), and rescale the output row in TMEM
-//              when the max has grown.
+//              when the max has grown.  The softmax's instruction stream is
+//              what the MMA issue competes with on every SM sub-partition, so
+//              it is kept short: a three-input max, packed two-lane fp32
+//              fma/add, and l summed from the fp32 weights before they are
+//              rounded to bf16 for P V (the quotient O / l then differs from
+//              one with l summed from the rounded weights by a relative
+//              2^-9 at most).
 // The rescale is lazy: the reference max m only moves when the tile max
 // exceeds it by more than 2^8, so P <= 256 and no value leaves fp32/bf16
 // range; the final O / l is the same quotient whichever reference max was
@@ -275,6 +281,35 @@ __device__ __forceinline__ void tmem_loaded(float *v) {
     for (int i = 0; i < N; ++i) asm volatile("" : "+f"(v[i]));
 }
 __device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+__device__ __forceinline__ uint64_t pack2(float lo, float hi) {
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+    return r;
+}
+__device__ __forceinline__ void unpack2(uint64_t v, float &lo, float &hi) {
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+// Two fp32 lanes at once (Blackwell packed FP32): a * b + c and a + b.
+__device__ __forceinline__ uint64_t fma2(uint64_t a, uint64_t b, uint64_t c) {
+    uint64_t r;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+    return r;
+}
+__device__ __forceinline__ uint64_t add2(uint64_t a, uint64_t b) {
+    uint64_t r;
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+__device__ __forceinline__ uint64_t mul2(uint64_t a, uint64_t b) {
+    uint64_t r;
+    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+__device__ __forceinline__ float max3(float a, float b, float c) {
+    float r;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+    return r;
+}
 __device__ __forceinline__ float ex2(float x) {
     float y;
     asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
@@ -548,7 +583,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         const bool row_valid = (tl < tpt) && (qt >= 0) && (tok0 + tl < Q);
         const int limit = row_valid ? (L - Q + tok0 + tl + 1) : kv_limit;
         const float sl2 = p.scale_log2;
-        float m_ref = -INFINITY, l = 0.f;
+        float m_ref = -INFINITY;
+        uint64_t l2 = pack2(0.f, 0.f);  // row sum, as two interleaved partial sums
         bool ok = true;
         for (int n = 0; n < ntiles; ++n) {
             const int b = n & 1;
@@ -570,7 +606,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             }
             float mx = sv[0];
 #pragma unroll
-            for (int i = 1; i < kKeys; ++i) mx = fmaxf(mx, sv[i]);
+            for (int i = 1; i + 1 < kKeys; i += 2) mx = max3(mx, sv[i], sv[i + 1]);
+            mx = fmaxf(mx, sv[kKeys - 1]);
             const float m_tile = mx * sl2;
             const bool grow = m_tile > m_ref + kRescaleLog2;  // always true on the first tile
             const float alpha = grow ? ex2(m_ref - m_tile) : 1.f;
@@ -591,9 +628,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                 tmem_wait_st();
             }
             if (grow) {
-                l *= alpha;
+                l2 = mul2(l2, pack2(alpha, alpha));
                 m_ref = m_tile;
             }
+            const uint64_t sl2x2 = pack2(sl2, sl2), nm2 = pack2(-m_ref, -m_ref);
             // P buffer b was last read by the P V of tile n - 2.
             if (n >= 2) {
                 if (!warp_wait(bar_pfree(b), ((n >> 1) - 1) & 1, abort, p.status)) { ok = false; break; }
@@ -607,10 +645,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 #pragma unroll
                 for (int e = 0; e < 16; ++e) {
                     const int i = c * 32 + 2 * e;
-                    const __nv_bfloat162 pr =
-                        __floats2bfloat162_rn(ex2(fmaf(sv[i], sl2, -m_ref)), ex2(fmaf(sv[i + 1], sl2, -m_ref)));
-                    const float2 back = __bfloat1622float2(pr);
-                    l += back.x + back.y;
+                    float x0, x1;
+                    unpack2(fma2(pack2(sv[i], sv[i + 1]), sl2x2, nm2), x0, x1);
+                    const float e0 = ex2(x0), e1 = ex2(x1);
+                    const __nv_bfloat162 pr = __floats2bfloat162_rn(e0, e1);
+                    l2 = add2(l2, pack2(e0, e1));
                     w[e] = *reinterpret_cast<const uint32_t *>(&pr);
                 }
                 tmem_st16u(trow + kColP + b * (kKeys / 2) + c * 16, w);
@@ -622,7 +661,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         }
         if (ok && warp_wait(bar_pfree((ntiles - 1) & 1), ((ntiles - 1) >> 1) & 1, abort, p.status)) {
             tc_fence_after();
-            const float inv = 1.f / l;
+            float la, lb;
+            unpack2(l2, la, lb);
+            const float inv = 1.f / (la + lb);
             uint16_t *orow = p.out + ((size_t)(qs0 + tok0 + tl) * p.num_q_heads + (size_t)j * g + hl) * kD;
 #pragma unroll
             for (int c = 0; c < 4; ++c) {
