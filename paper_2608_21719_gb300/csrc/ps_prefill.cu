@@ -52,6 +52,15 @@
 // range; the final O / l is the same quotient whichever reference max was
 // used.
 //
+// Persistent clusters.  A launch has one cluster per pair of SMs; each runs
+// a list of units -- (sequence, KV head, pair of query tiles) -- dealt out by
+// work (descending, in a snake over the clusters), with the rings, the S/P
+// buffers and their barrier phases running on from one unit to the next: the
+// next unit's Q (double-buffered) and first K/V tiles load while the current
+// unit finishes, and its first Q K^T runs while the softmax warps read out the
+// current unit's O.  (Batches with more units than fit a cluster's list run
+// one unit per cluster.)
+//
 // Every mbarrier wait gives up after ~2 s of globaltimer, or at once when
 // another role of its CTA has given up, and raises PS_DEVICE_TIMEOUT in the
 // optional device status word; the producers then wait for their own copies,
@@ -76,10 +85,10 @@ constexpr int kRows = 128;         // query rows per CTA (MMA M = 256 over the p
 constexpr int kKeys = 128;         // MMA N of S, K of P.V: keys per tile
 constexpr int kChunk = 16;         // keys per TMA box (one page slice)
 #ifndef PS_PREFILL_KSTAGES
-#define PS_PREFILL_KSTAGES 5
+#define PS_PREFILL_KSTAGES 4
 #endif
 #ifndef PS_PREFILL_VSTAGES
-#define PS_PREFILL_VSTAGES 5
+#define PS_PREFILL_VSTAGES 4
 #endif
 constexpr int kKStages = PS_PREFILL_KSTAGES;  // K ring: a stage is free once its Q K^T is done
 constexpr int kVStages = PS_PREFILL_VSTAGES;  // V ring: a stage is free once its P V is done
@@ -90,12 +99,19 @@ constexpr int kPairKeys = kKeys / 2;          // keys of each K tile one CTA hol
 constexpr int kKHalf = kPairKeys * 128;       // one 64-dim half of a CTA's K slice: 8 KiB
 constexpr int kKStage = 2 * kKHalf;           // 16 KiB
 constexpr int kVStage = kKeys * 128;          // 128 keys x this CTA's 64 dims: 16 KiB
-constexpr int kOffQ = 0;
-constexpr int kOffK = kOffQ + kQBytes;
+constexpr int kOffQ = 0;                            // two Q buffers: the next unit's Q loads early
+constexpr int kOffK = kOffQ + 2 * kQBytes;
 constexpr int kOffV = kOffK + kKStages * kKStage;
 constexpr int kOffBar = kOffV + kVStages * kVStage;
 constexpr int kBarBytes = 512;
-constexpr int kSmemBytes = 1024 + kOffBar + kBarBytes;  // 1 KiB of alignment slack
+constexpr int kMaxUnitsPerCluster = 256;            // a cluster's unit list (persistent mode)
+constexpr int kOffList = kOffBar + kBarBytes;
+constexpr int kSmemBytes = 1024 + kOffList + kMaxUnitsPerCluster * 4;  // 1 KiB of alignment slack
+// Persistent mode needs the whole batch's units (sequence x KV head x pair of
+// query tiles) below this; the host launches one unit per cluster above it.
+constexpr int kMaxPersistentUnits = 16384;
+constexpr int kSchedBins = 64;                      // work bins of the schedule's counting sort
+static_assert(kThreads * kSchedBins * 2 + 4 * kSchedBins * 4 <= kVStages * kVStage, "schedule scratch");
 static_assert(kSmemBytes <= 227 * 1024, "shared memory");
 constexpr uint32_t kTmemCols = 512;
 // TMEM columns (the same in both CTAs): S buffers at 0 and 128, O at 256, two
@@ -112,6 +128,8 @@ struct PrefillParams {
     int block_size, max_blocks_per_seq;
     long long num_blocks;
     float scale_log2;
+    int persistent;    // 1: grid of clusters, each running a list of units; 0: one unit per cluster
+    int num_clusters;  // persistent mode: clusters in the grid
 };
 
 // ------------------------------------------------------------ PTX wrappers --
@@ -345,6 +363,37 @@ __device__ __forceinline__ void drain_phase(uint32_t bar, uint32_t parity) {
 }
 
 
+// Geometry of unit u (sequence s, KV head j, pair pi of query tiles) and its
+// work in 128-key tiles; 0 for a unit with no query rows, or whose sequence is
+// inconsistent (then `bad` is set).
+struct Unit {
+    int s, j, qt_hi, qs0, Q, L, kv_limit, ntiles;
+};
+__device__ __forceinline__ Unit unit_of(const PrefillParams &p, int u, int npairs, bool &bad) {
+    Unit x;
+    const int pi = u % npairs;
+    x.j = (u / npairs) % p.num_kv_heads;
+    x.s = u / (npairs * p.num_kv_heads);
+    x.qt_hi = p.num_qtiles - 1 - 2 * pi;
+    x.qs0 = __ldg(p.q_start + x.s);
+    const int qs1 = __ldg(p.q_start + x.s + 1);
+    x.Q = qs1 - x.qs0;
+    x.L = __ldg(p.seq_lens + x.s);
+    x.ntiles = 0;
+    x.kv_limit = 0;
+    bad = false;
+    const int tpt = p.tokens_per_tile;
+    if (max(x.qt_hi - 1, 0) * tpt >= x.Q) return x;  // neither tile of the pair has rows
+    const long long cap = (long long)p.max_blocks_per_seq * p.block_size;
+    if (x.Q < 0 || x.L < x.Q || (long long)x.L > cap || x.qs0 < 0 || qs1 > p.total_q) {
+        bad = true;
+        return x;
+    }
+    x.kv_limit = x.L - x.Q + min(x.Q, (x.qt_hi + 1) * tpt);  // keys the pair needs: [0, kv_limit)
+    x.ntiles = (x.kv_limit + kKeys - 1) / kKeys;
+    return x;
+}
+
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     ps_prefill_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                       const __grid_constant__ CUtensorMap tmV, const PrefillParams p) {
@@ -352,39 +401,104 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const uint32_t rank = cta_rank();  // 0: the leader, which issues the MMAs
-    // Consecutive pairs share a (sequence, KV head), heaviest (last) query
-    // tiles first: the few K/V streams in flight at a time stay in L2.  The
-    // leader takes the later tile of its pair, the other CTA the one before
-    // (which may not exist: tile -1).
-    const int qt_hi = p.num_qtiles - 1 - 2 * (int)(blockIdx.x >> 1);
-    const int qt = qt_hi - (int)rank;
-    const int j = blockIdx.y, s = blockIdx.z;
     const int g = p.group, tpt = p.tokens_per_tile;
+    const int npairs = (p.num_qtiles + 1) / 2;
+    int *ulist = reinterpret_cast<int *>(sm + kOffList);
+    __shared__ int s_count, s_wmax;
 
-    // Sequence geometry (uniform over the pair).
-    const int qs0 = __ldg(p.q_start + s), qs1 = __ldg(p.q_start + s + 1);
-    const int Q = qs1 - qs0;
-    const int L = __ldg(p.seq_lens + s);
-    // max_q_len below a chunk leaves that chunk's later rows uncovered.
-    if (qt_hi == p.num_qtiles - 1 && rank == 0 && j == 0 && tid == 0 && Q > p.num_qtiles * tpt && p.status)
-        atomicOr(p.status, (unsigned)PS_DEVICE_LEN_CLAMPED);
-    if (max(qt_hi - 1, 0) * tpt >= Q) return;  // neither tile of the pair has rows
-    const long long cap = (long long)p.max_blocks_per_seq * p.block_size;
-    if (Q < 0 || L < Q || (long long)L > cap || qs0 < 0 || qs1 > p.total_q) {
-        if (tid == 0 && rank == 0 && j == 0 && p.status) atomicOr(p.status, (unsigned)PS_DEVICE_LEN_CLAMPED);
-        return;
+    // ---- the cluster's units ------------------------------------------
+    // One unit per cluster (grid order: heaviest pairs of query tiles first),
+    // or, in persistent mode, every cluster of the grid runs a list: all
+    // units sorted by work (descending, 64 bins, stable by unit index) and
+    // dealt out in a snake (0 .. P-1, P-1 .. 0, ...), so that the clusters'
+    // totals come out even.  Both CTAs of a cluster compute the same list.
+    if (!p.persistent) {
+        if (tid == 0) {
+            const int u = (blockIdx.z * p.num_kv_heads + blockIdx.y) * npairs + (blockIdx.x >> 1);
+            bool bad;
+            const Unit x = unit_of(p, u, npairs, bad);
+            if (bad && rank == 0 && p.status) atomicOr(p.status, (unsigned)PS_DEVICE_LEN_CLAMPED);
+            ulist[0] = u;
+            s_count = x.ntiles > 0 ? 1 : 0;
+        }
+    } else {
+        const int U = p.num_seqs * p.num_kv_heads * npairs;  // <= kMaxPersistentUnits (host)
+        const int P = p.num_clusters, me = (int)(blockIdx.x >> 1);
+        const int a = (int)((long long)tid * U / kThreads), e = (int)((long long)(tid + 1) * U / kThreads);
+        uint16_t *cnt = reinterpret_cast<uint16_t *>(sm + kOffV);                      // [kThreads][bins]
+        int *bin_start = reinterpret_cast<int *>(sm + kOffV + kThreads * kSchedBins * 2);  // [bins]
+        int *bin_total = bin_start + kSchedBins;
+        if (tid == 0) { s_wmax = 1; s_count = 0; }
+        for (int b = 0; b < kSchedBins; ++b) cnt[tid * kSchedBins + b] = 0;
+        __syncthreads();
+        int wmax = 1;
+        for (int u = a; u < e; ++u) {
+            bool bad;
+            const Unit x = unit_of(p, u, npairs, bad);
+            if (bad && blockIdx.x == 0 && p.status) atomicOr(p.status, (unsigned)PS_DEVICE_LEN_CLAMPED);
+            wmax = max(wmax, x.ntiles);
+        }
+        atomicMax(&s_wmax, wmax);
+        __syncthreads();
+        wmax = s_wmax;
+        auto bin_of = [&](int w) { return min(kSchedBins - 1, (int)((long long)(w - 1) * kSchedBins / wmax)); };
+        for (int u = a; u < e; ++u) {
+            bool bad;
+            const Unit x = unit_of(p, u, npairs, bad);
+            if (x.ntiles > 0) ++cnt[tid * kSchedBins + bin_of(x.ntiles)];
+        }
+        __syncthreads();
+        if (tid < kSchedBins) {  // per bin: units of earlier threads (stable by unit index)
+            int run = 0;
+            for (int t = 0; t < kThreads; ++t) {
+                const int c = cnt[t * kSchedBins + tid];
+                cnt[t * kSchedBins + tid] = (uint16_t)run;
+                run += c;
+            }
+            bin_total[tid] = run;
+        }
+        __syncthreads();
+        if (tid == 0) {  // bins in descending work
+            int acc = 0;
+            for (int b = kSchedBins - 1; b >= 0; --b) {
+                bin_start[b] = acc;
+                acc += bin_total[b];
+            }
+            const int full = acc / P, rem = acc - full * P;
+            s_count = full + ((full & 1) ? (P - 1 - me < rem) : (me < rem));
+        }
+        __syncthreads();
+        for (int u = a; u < e; ++u) {
+            bool bad;
+            const Unit x = unit_of(p, u, npairs, bad);
+            if (x.ntiles == 0) continue;
+            const int b = bin_of(x.ntiles);
+            const int r = bin_start[b] + cnt[tid * kSchedBins + b];
+            ++cnt[tid * kSchedBins + b];
+            const int round = r / P, pos = r - round * P;
+            if (((round & 1) ? P - 1 - pos : pos) == me) ulist[round] = u;
+        }
+        // max_q_len below a chunk leaves that chunk's later rows uncovered.
+        if (blockIdx.x == 0 && p.status)
+            for (int s = tid; s < p.num_seqs; s += kThreads)
+                if (__ldg(p.q_start + s + 1) - __ldg(p.q_start + s) > p.num_qtiles * tpt)
+                    atomicOr(p.status, (unsigned)PS_DEVICE_LEN_CLAMPED);
     }
-    const int tok0 = qt * tpt;                       // negative for the missing tile -1
-    const int kv_limit = L - Q + min(Q, (qt_hi + 1) * tpt);  // keys the pair needs: [0, kv_limit)
-    const int ntiles = (kv_limit + kKeys - 1) / kKeys;
+    if (!p.persistent && (blockIdx.x >> 1) == 0 && blockIdx.y == 0 && tid == 0 && rank == 0 && p.status) {
+        const int Qs = __ldg(p.q_start + blockIdx.z + 1) - __ldg(p.q_start + blockIdx.z);
+        if (Qs > p.num_qtiles * tpt) atomicOr(p.status, (unsigned)PS_DEVICE_LEN_CLAMPED);
+    }
+    __syncthreads();
+    const int nunits = s_count;  // the same in both CTAs of the cluster
+    if (nunits == 0) return;
 
     uint64_t *bars = reinterpret_cast<uint64_t *>(sm + kOffBar);
-    const uint32_t bar_q = saddr(bars + 0);
-    auto bar_kfull = [&](int st) { return saddr(bars + 1 + st); };                         // [kKStages], leader's
-    auto bar_kfree = [&](int st) { return saddr(bars + 1 + kKStages + st); };              // [kKStages]
-    auto bar_vfull = [&](int st) { return saddr(bars + 1 + 2 * kKStages + st); };          // [kVStages], leader's
-    auto bar_vfree = [&](int st) { return saddr(bars + 1 + 2 * kKStages + kVStages + st); };
-    constexpr int kB = 1 + 2 * kKStages + 2 * kVStages;
+    auto bar_q = [&](int qb) { return saddr(bars + qb); };                                    // [2] leader's
+    auto bar_kfull = [&](int st) { return saddr(bars + 2 + st); };                             // [kKStages], leader's
+    auto bar_kfree = [&](int st) { return saddr(bars + 2 + kKStages + st); };                  // [kKStages]
+    auto bar_vfull = [&](int st) { return saddr(bars + 2 + 2 * kKStages + st); };              // [kVStages], leader's
+    auto bar_vfree = [&](int st) { return saddr(bars + 2 + 2 * kKStages + kVStages + st); };
+    constexpr int kB = 2 + 2 * kKStages + 2 * kVStages;
     auto bar_sfull = [&](int b) { return saddr(bars + kB + b); };
     auto bar_sfree = [&](int b) { return saddr(bars + kB + 2 + b); };  // leader's
     auto bar_pfull = [&](int b) { return saddr(bars + kB + 4 + b); };  // leader's
@@ -393,10 +507,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     const uint32_t bar_vtail = saddr(bars + kB + 9);
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + kB + 10);
     volatile int *abort = reinterpret_cast<volatile int *>(bars + kB + 11);
-    static_assert((1 + 2 * kKStages + 2 * kVStages + 12) * 8 <= kBarBytes, "barrier area");
+    auto bar_qfree = [&](int qb) { return saddr(bars + kB + 12 + qb); };  // [2]
+    const uint32_t bar_ofree = saddr(bars + kB + 14);                     // leader's
+    static_assert((2 + 2 * kKStages + 2 * kVStages + 15) * 8 <= kBarBytes, "barrier area");
 
     if (tid == 0) {
-        mbar_init(bar_q, 2);  // one arrival (with its bytes) from each CTA
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(bar_q(i), 2);  // one arrival (with its bytes) from each CTA
+            mbar_init(bar_qfree(i), 1);
+        }
         for (int i = 0; i < kKStages; ++i) {
             mbar_init(bar_kfull(i), 2);
             mbar_init(bar_kfree(i), 1);
@@ -413,6 +532,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         }
         mbar_init(bar_mma_end, 1);
         mbar_init(bar_vtail, 1);
+        mbar_init(bar_ofree, 8);  // both CTAs' softmax warps have read O
         *abort = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -423,150 +543,176 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
     }
     // Both CTAs' barriers exist and their TMEM is allocated before either
-    // CTA's copies or arrivals can reach the other.
+    // CTA's copies or arrivals can reach the other (and the schedule scratch
+    // in the V ring is no longer read).
     tc_fence_before();
     cluster_sync();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
     const uint32_t sQ = saddr(sm + kOffQ), sK = saddr(sm + kOffK), sV = saddr(sm + kOffV);
+    bool bad_unused;
 
     if (warp == 0 || warp == 6) {
         // ----------------------------------------------------- producers --
         const bool is_k = warp == 0;
         uint64_t keep;  // every K/V page is read by all query tiles of its (sequence, head)
         asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(keep));
-        if (is_k && lane == 0) {
-            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmQ)) : "memory");
-            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmK)) : "memory");
-            const uint32_t lq = map_to(bar_q, 0);
-            mbar_expect_tx_cluster(lq, (uint32_t)(2 * 128 * g * tpt));
-            // Rows of a missing or empty tile read zeros or other rows; they are never written.
-            tma_load_3d_pair(sQ, &tmQ, 0, j * g, qs0 + tok0, lq, keep);
-            tma_load_3d_pair(sQ + kHalfQ, &tmQ, 64, j * g, qs0 + tok0, lq, keep);
+        if (lane == 0) {
+            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(is_k ? &tmK : &tmV)) : "memory");
+            if (is_k) asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmQ)) : "memory");
         }
-        if (!is_k && lane == 0)
-            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmV)) : "memory");
         const int stages = is_k ? kKStages : kVStages;
-        const int *bt_row = p.block_table + (size_t)s * p.max_blocks_per_seq;
-        int issued = 0;
-        bool tail_done = false;
-        for (int n = 0; n < ntiles; ++n) {
-            const int st = n % stages, use = n / stages;
-            if (n >= stages && !warp_wait(is_k ? bar_kfree(st) : bar_vfree(st), (use - 1) & 1, abort, p.status))
-                break;
-            const int base = n * kKeys;
+        int issued = 0, tails = 0, units_q = 0;
+        bool tail_pending = false, ok = true;
+        for (int ui = 0; ok && ui < nunits; ++ui) {
+            const Unit x = unit_of(p, ulist[ui], npairs, bad_unused);
+            const int qt = x.qt_hi - (int)rank, tok0 = qt * tpt;
+            const int *bt_row = p.block_table + (size_t)x.s * p.max_blocks_per_seq;
             if (is_k) {
-                // Keys 64 rank .. 64 rank + 63 of the tile, both 64-dim halves:
-                // lanes 0-7 take (chunk lane & 3, half lane >> 2).
-                const int k0 = base + kPairKeys * (int)rank;
-                const int nc = max(0, min(kPairKeys / kChunk, (kv_limit - k0 + kChunk - 1) / kChunk));
-                const uint32_t full = map_to(bar_kfull(st), 0);
-                if (lane == 0) mbar_expect_tx_cluster(full, (uint32_t)(nc * 2 * kChunk * 128));
-                __syncwarp();
-                const int c = lane & 3, half = lane >> 2;
-                if (lane < 8 && c < nc) {
-                    const int t0 = k0 + c * kChunk;
-                    const int lb = t0 / p.block_size;
-                    const int b = __ldg(bt_row + lb);
-                    int page = -1;  // out of range: TMA fills zeros
-                    if (b >= 0 && (long long)b < p.num_blocks) page = b * p.num_kv_heads + j;
-                    else if (p.status) atomicOr(p.status, (unsigned)PS_DEVICE_BAD_BLOCK);
-                    tma_load_3d_pair(sK + st * kKStage + half * kKHalf + c * (kChunk * 128), &tmK, half * 64,
-                                     t0 - lb * p.block_size, page, full, keep);
-                }
-            } else {
-                // Dims 64 rank .. 64 rank + 63 of all keys of the tile: lane c takes chunk c.
-                const int valid = min(kKeys, kv_limit - base);
-                const int nc = (valid + kChunk - 1) / kChunk;
-                const bool tail = valid < kKeys;
-                const uint32_t full = map_to(bar_vfull(st), 0);
+                // Q of this unit into buffer ui & 1, once the Q K^T of unit ui - 2 is done.
+                const int qb = ui & 1;
+                if (ui >= 2 && !warp_wait(bar_qfree(qb), ((ui - 2) >> 1) & 1, abort, p.status)) { ok = false; break; }
                 if (lane == 0) {
-                    if (tail) mbar_expect_tx(bar_vtail, (uint32_t)(nc * kChunk * 128));
-                    else mbar_expect_tx_cluster(full, (uint32_t)(nc * kChunk * 128));
+                    const uint32_t lq = map_to(bar_q(qb), 0);
+                    mbar_expect_tx_cluster(lq, (uint32_t)(2 * 128 * g * tpt));
+                    // Rows of a missing or empty tile read zeros or other rows; they are never written.
+                    tma_load_3d_pair(sQ + qb * kQBytes, &tmQ, 0, x.j * g, x.qs0 + tok0, lq, keep);
+                    tma_load_3d_pair(sQ + qb * kQBytes + kHalfQ, &tmQ, 64, x.j * g, x.qs0 + tok0, lq, keep);
                 }
-                __syncwarp();
-                if (lane < nc) {
-                    const int t0 = base + lane * kChunk;
-                    const int lb = t0 / p.block_size;
-                    const int b = __ldg(bt_row + lb);
-                    int page = -1;
-                    if (b >= 0 && (long long)b < p.num_blocks) page = b * p.num_kv_heads + j;
-                    const uint32_t dst = sV + st * kVStage + lane * (kChunk * 128);
-                    if (tail) tma_load_3d_hint(dst, &tmV, 64 * (int)rank, t0 - lb * p.block_size, page, bar_vtail, keep);
-                    else tma_load_3d_pair(dst, &tmV, 64 * (int)rank, t0 - lb * p.block_size, page, full, keep);
-                }
-                issued = n + 1;
-                if (tail) {
-                    // The last tile: its copy completes here first, then the rows
-                    // past the needed keys (other tokens' data, or stale bytes)
-                    // are zeroed -- P is zero there -- before the leader is told.
-                    if (!warp_wait(bar_vtail, 0, abort, p.status)) break;
-                    tail_done = true;
-                    uint8_t *v = sm + kOffV + st * kVStage;
-                    for (int e = lane; e < (kKeys - valid) * 8; e += 32)
-                        *reinterpret_cast<uint4 *>(v + (valid + (e >> 3)) * 128 + (e & 7) * 16) = make_uint4(0, 0, 0, 0);
-                    fence_proxy_async_smem();
+                units_q = ui + 1;
+            }
+            for (int n = 0; n < x.ntiles; ++n) {
+                const int st = issued % stages, use = issued / stages;
+                if (issued >= stages &&
+                    !warp_wait(is_k ? bar_kfree(st) : bar_vfree(st), (use - 1) & 1, abort, p.status)) { ok = false; break; }
+                const int base = n * kKeys;
+                if (is_k) {
+                    // Keys 64 rank .. 64 rank + 63 of the tile, both 64-dim halves:
+                    // lanes 0-7 take (chunk lane & 3, half lane >> 2).
+                    const int k0 = base + kPairKeys * (int)rank;
+                    const int nc = max(0, min(kPairKeys / kChunk, (x.kv_limit - k0 + kChunk - 1) / kChunk));
+                    const uint32_t full = map_to(bar_kfull(st), 0);
+                    if (lane == 0) mbar_expect_tx_cluster(full, (uint32_t)(nc * 2 * kChunk * 128));
                     __syncwarp();
-                    if (lane == 0) mbar_arrive_cluster(full);
+                    const int c = lane & 3, half = lane >> 2;
+                    if (lane < 8 && c < nc) {
+                        const int t0 = k0 + c * kChunk;
+                        const int lb = t0 / p.block_size;
+                        const int b = __ldg(bt_row + lb);
+                        int page = -1;  // out of range: TMA fills zeros
+                        if (b >= 0 && (long long)b < p.num_blocks) page = b * p.num_kv_heads + x.j;
+                        else if (p.status) atomicOr(p.status, (unsigned)PS_DEVICE_BAD_BLOCK);
+                        tma_load_3d_pair(sK + st * kKStage + half * kKHalf + c * (kChunk * 128), &tmK, half * 64,
+                                         t0 - lb * p.block_size, page, full, keep);
+                    }
+                    ++issued;
+                } else {
+                    // Dims 64 rank .. 64 rank + 63 of all keys of the tile: lane c takes chunk c.
+                    const int valid = min(kKeys, x.kv_limit - base);
+                    const int nc = (valid + kChunk - 1) / kChunk;
+                    const bool tail = valid < kKeys;
+                    const uint32_t full = map_to(bar_vfull(st), 0);
+                    if (lane == 0) {
+                        if (tail) mbar_expect_tx(bar_vtail, (uint32_t)(nc * kChunk * 128));
+                        else mbar_expect_tx_cluster(full, (uint32_t)(nc * kChunk * 128));
+                    }
+                    __syncwarp();
+                    if (lane < nc) {
+                        const int t0 = base + lane * kChunk;
+                        const int lb = t0 / p.block_size;
+                        const int b = __ldg(bt_row + lb);
+                        int page = -1;
+                        if (b >= 0 && (long long)b < p.num_blocks) page = b * p.num_kv_heads + x.j;
+                        const uint32_t dst = sV + st * kVStage + lane * (kChunk * 128);
+                        if (tail) tma_load_3d_hint(dst, &tmV, 64 * (int)rank, t0 - lb * p.block_size, page, bar_vtail, keep);
+                        else tma_load_3d_pair(dst, &tmV, 64 * (int)rank, t0 - lb * p.block_size, page, full, keep);
+                    }
+                    ++issued;
+                    if (tail) {
+                        // The unit's last tile: its copy completes here first, then the
+                        // rows past the needed keys (other tokens' data, or stale bytes)
+                        // are zeroed -- P is zero there -- before the leader is told.
+                        tail_pending = true;
+                        if (!warp_wait(bar_vtail, tails & 1, abort, p.status)) { ok = false; break; }
+                        tail_pending = false;
+                        ++tails;
+                        uint8_t *v = sm + kOffV + st * kVStage;
+                        for (int e2 = lane; e2 < (kKeys - valid) * 8; e2 += 32)
+                            *reinterpret_cast<uint4 *>(v + (valid + (e2 >> 3)) * 128 + (e2 & 7) * 16) = make_uint4(0, 0, 0, 0);
+                        fence_proxy_async_smem();
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive_cluster(full);
+                    }
                 }
             }
-            issued = n + 1;
         }
         // Drain: this CTA's copies must land before it can leave.  Copies that
         // count on the leader's barriers are covered by the leader's waits and
         // the final cluster barrier; the local ones are waited for here.
-        if (!is_k && !tail_done && issued > 0 && min(kKeys, kv_limit - (issued - 1) * kKeys) < kKeys)
-            drain_phase(bar_vtail, 0);
+        if (tail_pending) drain_phase(bar_vtail, tails & 1);
         if (rank == 0) {
-            for (int n = max(0, issued - stages); n < issued; ++n)
-                drain_phase(is_k ? bar_kfull(n % stages) : bar_vfull(n % stages), (n / stages) & 1);
-            if (is_k) drain_phase(bar_q, 0);
+            for (int i = max(0, issued - stages); i < issued; ++i)
+                drain_phase(is_k ? bar_kfull(i % stages) : bar_vfull(i % stages), (i / stages) & 1);
+            if (is_k)
+                for (int ui = max(0, units_q - 2); ui < units_q; ++ui) drain_phase(bar_q(ui & 1), (ui >> 1) & 1);
         }
     } else if (warp == 1) {
         if (rank == 0) {
             // ---------------------------------------- MMA issuer (leader) --
             constexpr uint32_t idS = instr_desc(2 * kRows, kKeys, 0);
             constexpr uint32_t idO = instr_desc(2 * kRows, kD, 1);
-            bool ok = warp_wait(bar_q, 0, abort, p.status);
             // Descriptor bases, once: a stage or K-step offset is an add to the
             // 14-bit start-address field (shared-memory addresses stay below 256 KiB).
             const uint64_t dQ = smem_desc(sQ, 16, 1024), dK = smem_desc(sK, 16, 1024), dV = smem_desc(sV, 16, 1024);
-            for (int n = 0; ok && n <= ntiles; ++n) {
-                if (n < ntiles) {
-                    const int st = n % kKStages, b = n & 1;
-                    if (!warp_wait(bar_kfull(st), (n / kKStages) & 1, abort, p.status)) { ok = false; break; }
-                    if (n >= 2 && !warp_wait(bar_sfree(b), ((n >> 1) - 1) & 1, abort, p.status)) { ok = false; break; }
-                    tc_fence_after();
-                    if (lane == 0) {
-                        const uint64_t kd = dK + (uint64_t)((st * kKStage) >> 4);
+            bool ok = true;
+            int t0 = 0;  // tiles of the earlier units (S/P buffers and K/V stages run on across units)
+            for (int ui = 0; ok && ui < nunits; ++ui) {
+                const Unit x = unit_of(p, ulist[ui], npairs, bad_unused);
+                const int qb = ui & 1;
+                if (!warp_wait(bar_q(qb), (ui >> 1) & 1, abort, p.status)) { ok = false; break; }
+                const uint64_t dq = dQ + (uint64_t)((qb * kQBytes) >> 4);
+                for (int n = 0; ok && n <= x.ntiles; ++n) {
+                    if (n < x.ntiles) {
+                        const int t = t0 + n, st = t % kKStages, b = t & 1;
+                        if (!warp_wait(bar_kfull(st), (t / kKStages) & 1, abort, p.status)) { ok = false; break; }
+                        if (t >= 2 && !warp_wait(bar_sfree(b), ((t >> 1) - 1) & 1, abort, p.status)) { ok = false; break; }
+                        tc_fence_after();
+                        if (lane == 0) {
+                            const uint64_t kd = dK + (uint64_t)((st * kKStage) >> 4);
 #pragma unroll
-                        for (int kk = 0; kk < kD / 16; ++kk) {
-                            umma2(tmem + b * kKeys, dQ + (uint64_t)(((kk >> 2) * kHalfQ + (kk & 3) * 32) >> 4),
-                                  kd + (uint64_t)(((kk >> 2) * kKHalf + (kk & 3) * 32) >> 4), idS, kk > 0);
+                            for (int kk = 0; kk < kD / 16; ++kk) {
+                                umma2(tmem + b * kKeys, dq + (uint64_t)(((kk >> 2) * kHalfQ + (kk & 3) * 32) >> 4),
+                                      kd + (uint64_t)(((kk >> 2) * kKHalf + (kk & 3) * 32) >> 4), idS, kk > 0);
+                            }
+                            umma_commit_pair(bar_sfull(b));
+                            umma_commit_pair(bar_kfree(st));
+                            if (n == x.ntiles - 1) umma_commit_pair(bar_qfree(qb));  // Q buffer qb is free again
                         }
-                        umma_commit_pair(bar_sfull(b));
-                        umma_commit_pair(bar_kfree(st));
+                        __syncwarp();
                     }
-                    __syncwarp();
-                }
-                if (n >= 1) {
-                    const int m = n - 1, st = m % kVStages;
-                    if (!warp_wait(bar_vfull(st), (m / kVStages) & 1, abort, p.status)) { ok = false; break; }
-                    if (!warp_wait(bar_pfull(m & 1), (m >> 1) & 1, abort, p.status)) { ok = false; break; }
-                    tc_fence_after();
-                    if (lane == 0) {
-                        const uint32_t pt = tmem + kColP + (m & 1) * (kKeys / 2);
-                        const uint64_t vd = dV + (uint64_t)((st * kVStage) >> 4);
+                    if (n >= 1) {
+                        const int m = n - 1, t = t0 + m, st = t % kVStages;
+                        if (!warp_wait(bar_vfull(st), (t / kVStages) & 1, abort, p.status)) { ok = false; break; }
+                        if (!warp_wait(bar_pfull(t & 1), (t >> 1) & 1, abort, p.status)) { ok = false; break; }
+                        // The unit's first P V overwrites O: the previous unit's O must
+                        // have been read out by both CTAs' softmax warps.
+                        if (m == 0 && ui > 0 && !warp_wait(bar_ofree, (ui - 1) & 1, abort, p.status)) { ok = false; break; }
+                        tc_fence_after();
+                        if (lane == 0) {
+                            const uint32_t pt = tmem + kColP + (t & 1) * (kKeys / 2);
+                            const uint64_t vd = dV + (uint64_t)((st * kVStage) >> 4);
 #pragma unroll
-                        for (int kk = 0; kk < kKeys / 16; ++kk)
-                            umma2_ts(tmem + kColO, pt + kk * 8, vd + (uint64_t)((kk * (16 * 128)) >> 4), idO,
-                                     (m > 0 || kk > 0) ? 1u : 0u);
-                        umma_commit_pair(bar_pfree(m & 1));
-                        umma_commit_pair(bar_vfree(st));
+                            for (int kk = 0; kk < kKeys / 16; ++kk)
+                                umma2_ts(tmem + kColO, pt + kk * 8, vd + (uint64_t)((kk * (16 * 128)) >> 4), idO,
+                                         (m > 0 || kk > 0) ? 1u : 0u);
+                            umma_commit_pair(bar_pfree(t & 1));
+                            umma_commit_pair(bar_vfree(st));
+                        }
+                        __syncwarp();
                     }
-                    __syncwarp();
                 }
+                t0 += x.ntiles;
             }
             // Every MMA issued above has finished, in both CTAs, before TMEM
             // and shared memory go away.
@@ -580,110 +726,120 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         const int r = quarter * 32 + lane;
         const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
         const int tl = r / g, hl = r - tl * g;
-        const bool row_valid = (tl < tpt) && (qt >= 0) && (tok0 + tl < Q);
-        const int limit = row_valid ? (L - Q + tok0 + tl + 1) : kv_limit;
         const float sl2 = p.scale_log2;
-        float m_ref = -INFINITY;
-        uint64_t l2 = pack2(0.f, 0.f);  // row sum, as two interleaved partial sums
         bool ok = true;
-        for (int n = 0; n < ntiles; ++n) {
-            const int b = n & 1;
-            if (!warp_wait(bar_sfull(b), (n >> 1) & 1, abort, p.status)) { ok = false; break; }
-            tc_fence_after();
-            float sv[kKeys];
-#pragma unroll
-            for (int c = 0; c < 4; ++c) tmem_ld32(trow + b * kKeys + c * 32, sv + c * 32);
-            tmem_wait_ld();
-            tmem_loaded<kKeys>(sv);
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive_cluster(map_to(bar_sfree(b), 0));
-            const int base = n * kKeys;
-            if (base + kKeys > limit) {
-#pragma unroll
-                for (int i = 0; i < kKeys; ++i)
-                    if (base + i >= limit) sv[i] = -INFINITY;
-            }
-            float mx = sv[0];
-#pragma unroll
-            for (int i = 1; i + 1 < kKeys; i += 2) mx = max3(mx, sv[i], sv[i + 1]);
-            mx = fmaxf(mx, sv[kKeys - 1]);
-            const float m_tile = mx * sl2;
-            const bool grow = m_tile > m_ref + kRescaleLog2;  // always true on the first tile
-            const float alpha = grow ? ex2(m_ref - m_tile) : 1.f;
-            if (n >= 1 && __any_sync(0xffffffffu, grow)) {
-                // O must hold key tiles 0 .. n-1 before it is rescaled.
-                if (!warp_wait(bar_pfree((n - 1) & 1), ((n - 1) >> 1) & 1, abort, p.status)) { ok = false; break; }
+        int t0 = 0;
+        for (int ui = 0; ok && ui < nunits; ++ui) {
+            const Unit x = unit_of(p, ulist[ui], npairs, bad_unused);
+            const int qt = x.qt_hi - (int)rank, tok0 = qt * tpt;
+            const bool row_valid = (tl < tpt) && (qt >= 0) && (tok0 + tl < x.Q);
+            const int limit = row_valid ? (x.L - x.Q + tok0 + tl + 1) : x.kv_limit;
+            float m_ref = -INFINITY;
+            uint64_t l2 = pack2(0.f, 0.f);  // row sum, as two interleaved partial sums
+            for (int n = 0; n < x.ntiles; ++n) {
+                const int t = t0 + n, b = t & 1;
+                if (!warp_wait(bar_sfull(b), (t >> 1) & 1, abort, p.status)) { ok = false; break; }
                 tc_fence_after();
+                float sv[kKeys];
+#pragma unroll
+                for (int c = 0; c < 4; ++c) tmem_ld32(trow + b * kKeys + c * 32, sv + c * 32);
+                tmem_wait_ld();
+                tmem_loaded<kKeys>(sv);
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive_cluster(map_to(bar_sfree(b), 0));
+                const int base = n * kKeys;
+                if (base + kKeys > limit) {
+#pragma unroll
+                    for (int i = 0; i < kKeys; ++i)
+                        if (base + i >= limit) sv[i] = -INFINITY;
+                }
+                float mx = sv[0];
+#pragma unroll
+                for (int i = 1; i + 1 < kKeys; i += 2) mx = max3(mx, sv[i], sv[i + 1]);
+                mx = fmaxf(mx, sv[kKeys - 1]);
+                const float m_tile = mx * sl2;
+                const bool grow = m_tile > m_ref + kRescaleLog2;  // always true on a unit's first tile
+                const float alpha = grow ? ex2(m_ref - m_tile) : 1.f;
+                if (n >= 1 && __any_sync(0xffffffffu, grow)) {
+                    // O must hold key tiles 0 .. n-1 before it is rescaled.
+                    if (!warp_wait(bar_pfree((t - 1) & 1), ((t - 1) >> 1) & 1, abort, p.status)) { ok = false; break; }
+                    tc_fence_after();
+#pragma unroll
+                    for (int c = 0; c < 4; ++c) {
+                        float ov[32];
+                        tmem_ld32(trow + kColO + c * 32, ov);
+                        tmem_wait_ld();
+                        tmem_loaded<32>(ov);
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) ov[i] *= alpha;
+                        tmem_st32(trow + kColO + c * 32, ov);
+                    }
+                    tmem_wait_st();
+                }
+                if (grow) {
+                    l2 = mul2(l2, pack2(alpha, alpha));
+                    m_ref = m_tile;
+                }
+                const uint64_t sl2x2 = pack2(sl2, sl2), nm2 = pack2(-m_ref, -m_ref);
+                // P buffer b was last read by the P V of tile t - 2.
+                if (t >= 2) {
+                    if (!warp_wait(bar_pfree(b), ((t >> 1) - 1) & 1, abort, p.status)) { ok = false; break; }
+                    tc_fence_after();
+                }
+                // P row (bf16 pairs) into TMEM buffer b, row = this thread's lane:
+                // the A operand of the P V MMA.
 #pragma unroll
                 for (int c = 0; c < 4; ++c) {
-                    float ov[32];
-                    tmem_ld32(trow + kColO + c * 32, ov);
-                    tmem_wait_ld();
-                    tmem_loaded<32>(ov);
+                    uint32_t w[16];
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) ov[i] *= alpha;
-                    tmem_st32(trow + kColO + c * 32, ov);
+                    for (int e = 0; e < 16; ++e) {
+                        const int i = c * 32 + 2 * e;
+                        float x0, x1;
+                        unpack2(fma2(pack2(sv[i], sv[i + 1]), sl2x2, nm2), x0, x1);
+                        const float e0 = ex2(x0), e1 = ex2(x1);
+                        const __nv_bfloat162 pr = __floats2bfloat162_rn(e0, e1);
+                        l2 = add2(l2, pack2(e0, e1));
+                        w[e] = *reinterpret_cast<const uint32_t *>(&pr);
+                    }
+                    tmem_st16u(trow + kColP + b * (kKeys / 2) + c * 16, w);
                 }
                 tmem_wait_st();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive_cluster(map_to(bar_pfull(b), 0));
             }
-            if (grow) {
-                l2 = mul2(l2, pack2(alpha, alpha));
-                m_ref = m_tile;
-            }
-            const uint64_t sl2x2 = pack2(sl2, sl2), nm2 = pack2(-m_ref, -m_ref);
-            // P buffer b was last read by the P V of tile n - 2.
-            if (n >= 2) {
-                if (!warp_wait(bar_pfree(b), ((n >> 1) - 1) & 1, abort, p.status)) { ok = false; break; }
-                tc_fence_after();
-            }
-            // P row (bf16 pairs) into TMEM buffer b, row = this thread's lane:
-            // the A operand of the P V MMA.
+            if (!ok) break;
+            const int tl_last = t0 + x.ntiles - 1;
+            if (!warp_wait(bar_pfree(tl_last & 1), (tl_last >> 1) & 1, abort, p.status)) { ok = false; break; }
+            tc_fence_after();
+            // O of this unit into registers, then the leader may start the next
+            // unit's P V (which overwrites O) while the rows are written out.
+            float ov[kD];
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                uint32_t w[16];
-#pragma unroll
-                for (int e = 0; e < 16; ++e) {
-                    const int i = c * 32 + 2 * e;
-                    float x0, x1;
-                    unpack2(fma2(pack2(sv[i], sv[i + 1]), sl2x2, nm2), x0, x1);
-                    const float e0 = ex2(x0), e1 = ex2(x1);
-                    const __nv_bfloat162 pr = __floats2bfloat162_rn(e0, e1);
-                    l2 = add2(l2, pack2(e0, e1));
-                    w[e] = *reinterpret_cast<const uint32_t *>(&pr);
-                }
-                tmem_st16u(trow + kColP + b * (kKeys / 2) + c * 16, w);
-            }
-            tmem_wait_st();
+            for (int c = 0; c < 4; ++c) tmem_ld32(trow + kColO + c * 32, ov + c * 32);
+            tmem_wait_ld();
+            tmem_loaded<kD>(ov);
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive_cluster(map_to(bar_pfull(b), 0));
-        }
-        if (ok && warp_wait(bar_pfree((ntiles - 1) & 1), ((ntiles - 1) >> 1) & 1, abort, p.status)) {
-            tc_fence_after();
+            if (lane == 0) mbar_arrive_cluster(map_to(bar_ofree, 0));
             float la, lb;
             unpack2(l2, la, lb);
             const float inv = 1.f / (la + lb);
-            uint16_t *orow = p.out + ((size_t)(qs0 + tok0 + tl) * p.num_q_heads + (size_t)j * g + hl) * kD;
+            if (row_valid) {
+                uint16_t *orow = p.out + ((size_t)(x.qs0 + tok0 + tl) * p.num_q_heads + (size_t)x.j * g + hl) * kD;
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                float ov[32];
-                tmem_ld32(trow + kColO + c * 32, ov);
-                tmem_wait_ld();
-                tmem_loaded<32>(ov);
-                if (row_valid) {
+                for (int v = 0; v < kD / 8; ++v) {
+                    uint32_t w[4];
 #pragma unroll
-                    for (int v = 0; v < 4; ++v) {
-                        uint32_t w[4];
-#pragma unroll
-                        for (int e = 0; e < 4; ++e) {
-                            const __nv_bfloat162 pr = __floats2bfloat162_rn(ov[v * 8 + 2 * e] * inv, ov[v * 8 + 2 * e + 1] * inv);
-                            w[e] = *reinterpret_cast<const uint32_t *>(&pr);
-                        }
-                        *reinterpret_cast<uint4 *>(orow + c * 32 + v * 8) = make_uint4(w[0], w[1], w[2], w[3]);
+                    for (int e = 0; e < 4; ++e) {
+                        const __nv_bfloat162 pr = __floats2bfloat162_rn(ov[v * 8 + 2 * e] * inv, ov[v * 8 + 2 * e + 1] * inv);
+                        w[e] = *reinterpret_cast<const uint32_t *>(&pr);
                     }
+                    *reinterpret_cast<uint4 *>(orow + v * 8) = make_uint4(w[0], w[1], w[2], w[3]);
                 }
             }
+            t0 += x.ntiles;
         }
     }
     // Neither CTA leaves (nor frees TMEM) while the other may still touch its
@@ -787,8 +943,19 @@ extern "C" ps_status_t ps_prefill_attention(const void *q, const void *k_cache, 
     pp.max_blocks_per_seq = max_blocks_per_seq;
     pp.num_blocks = num_blocks;
     pp.scale_log2 = scale * 1.4426950408889634f;
-    // Clusters of two CTAs, one pair per two adjacent query tiles.
-    const dim3 grid((unsigned)(2 * ((nqt + 1) / 2)), (unsigned)num_kv_heads, (unsigned)num_seqs);
+    // Units: (sequence, KV head, pair of adjacent query tiles).  Up to
+    // kMaxPersistentUnits of them, one cluster of two CTAs per pair of SMs
+    // runs a list of units (persistent); beyond, one cluster per unit.
+    const long long npairs = (nqt + 1) / 2;
+    const long long units = (long long)num_seqs * num_kv_heads * npairs;
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+        return PS_ERR_CUDA;
+    const int clusters = max(1, sms / 2);
+    pp.persistent = (units <= kMaxPersistentUnits && (units + clusters - 1) / clusters <= kMaxUnitsPerCluster) ? 1 : 0;
+    pp.num_clusters = clusters;
+    const dim3 grid = pp.persistent ? dim3((unsigned)(2 * clusters), 1, 1)
+                                    : dim3((unsigned)(2 * npairs), (unsigned)num_kv_heads, (unsigned)num_seqs);
     if (ps::take_injected_launch_error() != cudaSuccess) return PS_ERR_CUDA;
     ps_prefill_kernel<<<grid, kThreads, kSmemBytes, reinterpret_cast<cudaStream_t>(stream)>>>(tmQ, tmK, tmV, pp);
     if (cudaGetLastError() != cudaSuccess) return PS_ERR_CUDA;

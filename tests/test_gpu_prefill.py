@@ -182,6 +182,21 @@ def test_full_size_prefill_every_row(psd):
     _compare(out, _oracle(wl), "p2, all %d outputs" % out.numel(), rel=0.0)
 
 
+def test_prefill_with_more_units_than_a_persistent_launch_holds(psd):
+    """Above 16384 units (sequence x KV head x pair of query tiles) the kernel
+    runs one unit per cluster instead of persistent clusters: 2100 short
+    chunks x 8 KV heads (16800 units), every output against the oracle."""
+    rng = np.random.default_rng(31)
+    new = rng.integers(1, 33, size=2100)  # one query-tile pair per sequence at g = 4
+    prior = rng.integers(0, 60, size=2100)
+    wl = inputs.make_prefill_workload("p1", device="cpu", new=new, prior=prior, num_q_heads=32, num_kv_heads=8,
+                                      seed=31).to("cuda")
+    assert wl.seq_lens.shape[0] * 8 * ((wl.max_q_len + 31) // 32 + 1) // 2 > 16384
+    out, status = _gpu(psd, wl)
+    assert status == 0
+    _compare(out, _oracle(wl), "16800 units")
+
+
 def test_prefill_counts_one_launch_per_call(psd):
     wl = inputs.make_prefill_workload("p1", device="cpu", new=[50, 20], prior=[10, 300]).to("cuda")
     before = psd.ps_decode_launch_count()
