@@ -25,40 +25,53 @@
 // a pair stream the keys the later tile needs; the earlier tile masks the
 // rest.
 //
-// Per key tile n (warp roles, 7 warps per CTA):
-//   warp 0     TMA: Q once, then this CTA's half of K_n into a K ring.
-//   warp 6     TMA: this CTA's half of V_n into a V ring; the last tile's rows
-//              past the needed keys are zeroed (its copy completes locally
-//              first) before the leader is told.
-//   warp 1     leader CTA only, one thread: S_n = Q K_n^T into one of two TMEM
-//              score buffers of both CTAs (M = 256, N = 128, K = 128), then,
-//              once both CTAs' softmax has written P_{n-1}, O += P_{n-1}
-//              V_{n-1} with P read from TMEM; tcgen05.commit multicasts each
-//              completion to both CTAs' barriers.
-//   warps 2-5  softmax, one TMEM lane (= one row) per thread, in each CTA:
-//              load the score row, mask it causally, update the running max
-//              m and sum l in fp32 (base 2, log2 e folded into the scale),
-//              write the bf16 probabilities into TMEM P buffer n & 1 (the A
-//              operand of the P V MMA), and rescale the output row in TMEM
-//              when the max has grown.  The softmax's instruction stream is
-//              what the MMA issue competes with on every SM sub-partition, so
-//              it is kept short: a three-input max, packed two-lane fp32
-//              fma/add, and l summed from the fp32 weights before they are
-//              rounded to bf16 for P V (the quotient O / l then differs from
-//              one with l summed from the rounded weights by a relative
-//              2^-9 at most).
-// The rescale is lazy: the reference max m only moves when the tile max
-// exceeds it by more than 2^8, so P <= 256 and no value leaves fp32/bf16
+// Warp roles (12 warps per CTA; warpgroup 0 gives registers to the two
+// softmax warpgroups with setmaxnreg, 56 / 224 per thread):
+//   warp 0     TMA: Q once per unit, then this CTA's half of each K tile into
+//              a K ring.
+//   warp 2     TMA: this CTA's half of each V tile into a V ring; the last
+//              tile's rows past the needed keys are zeroed (its copy completes
+//              locally first) before the leader is told.
+//   warp 1     leader CTA only, one thread: S_n = Q K_n^T into TMEM score
+//              buffer n & 1 of both CTAs (M = 256, N = 128, K = 128), and, once
+//              both CTAs' softmax has written P_n, O_{n & 1} += P_n V_n with P
+//              read from TMEM; tcgen05.commit multicasts each completion to
+//              both CTAs' barriers.
+//   warp 3     idle (completes warpgroup 0).
+//   warps 4-7  softmax group 0: the tiles of even global index n;
+//   warps 8-11 softmax group 1: the tiles of odd n.  One TMEM lane (= one
+//              row) per thread: load the score row, mask it causally, update
+//              the running max m and sum l in fp32 (base 2, log2 e folded into
+//              the scale), and write the bf16 probabilities over the first
+//              half of the same S buffer (the A operand of the P V MMA).
+// Each group thus runs an independent online softmax over every other key
+// tile with its own accumulator (TMEM: S_0, S_1 at columns 0 and 128, O_0,
+// O_1 at 256 and 384), so that one group computes while the other waits for
+// its next score tile and the tensor core works on both: two softmax streams
+// per SM sub-partition where one left the sub-partition idle during every
+// wait.  At the end of a unit group 1 hands (m, l) of each row to group 0
+// through shared memory and group 0 merges the halves -- O = (2^(m_0 - m) O_0
+// + 2^(m_1 - m) O_1) / (2^(m_0 - m) l_0 + 2^(m_1 - m) l_1), m = max(m_0, m_1)
+// -- and writes the row.  P over S needs no barrier of its own: the Q K^T of
+// tile n + 2 is issued after the P V of tile n, and tcgen05 MMAs of one
+// thread run in order.  The softmax's instruction stream is what the MMA
+// issue competes with on every SM sub-partition, so it is kept short: a
+// three-input max, packed two-lane fp32 fma/add, and l summed from the fp32
+// weights before they are rounded to bf16 for P V (the quotient O / l then
+// differs from one with l summed from the rounded weights by a relative 2^-9
+// at most).
+// The rescale is lazy: a group's reference max m only moves when the tile
+// max exceeds it by more than 2^8, so P <= 256 and no value leaves fp32/bf16
 // range; the final O / l is the same quotient whichever reference max was
 // used.
-//
+
 // Persistent clusters.  A launch has one cluster per pair of SMs; each runs
 // a list of units -- (sequence, KV head, pair of query tiles) -- dealt out by
 // work (descending, in a snake over the clusters), with the rings, the S/P
 // buffers and their barrier phases running on from one unit to the next: the
 // next unit's Q (double-buffered) and first K/V tiles load while the current
-// unit finishes, and its first Q K^T runs while the softmax warps read out the
-// current unit's O.  (Batches with more units than fit a cluster's list run
+// unit finishes, and its first Q K^T runs while softmax group 0 merges and
+// writes out the current unit's rows.  (Batches with more units than fit a cluster's list run
 // one unit per cluster.)
 //
 // Every mbarrier wait gives up after ~2 s of globaltimer, or at once when
@@ -92,7 +105,13 @@ constexpr int kChunk = 16;         // keys per TMA box (one page slice)
 #endif
 constexpr int kKStages = PS_PREFILL_KSTAGES;  // K ring: a stage is free once its Q K^T is done
 constexpr int kVStages = PS_PREFILL_VSTAGES;  // V ring: a stage is free once its P V is done
-constexpr int kThreads = 224;
+constexpr int kThreads = 384;
+// Registers per thread after the role split: warpgroup 0 (producers, MMA
+// issuer) gives registers back, the two softmax warpgroups take them.  The sum
+// must not exceed what the block is launched with (kThreads x the kernel's
+// register count, checked on the host), or setmaxnreg.inc would wait forever.
+constexpr int kRegsCtl = 56, kRegsSoftmax = 224;
+static_assert(128 * kRegsCtl + 256 * kRegsSoftmax <= 65536, "register split");
 constexpr int kHalfQ = kRows * 64 * 2;        // one 64-column half of the 128-row Q tile: 16 KiB
 constexpr int kQBytes = 2 * kHalfQ;           // 32 KiB
 constexpr int kPairKeys = kKeys / 2;          // keys of each K tile one CTA holds
@@ -106,7 +125,8 @@ constexpr int kOffBar = kOffV + kVStages * kVStage;
 constexpr int kBarBytes = 512;
 constexpr int kMaxUnitsPerCluster = 256;            // a cluster's unit list (persistent mode)
 constexpr int kOffList = kOffBar + kBarBytes;
-constexpr int kSmemBytes = 1024 + kOffList + kMaxUnitsPerCluster * 4;  // 1 KiB of alignment slack
+constexpr int kOffX = kOffList + kMaxUnitsPerCluster * 4;  // (m, l) of group 1 rows for the merge
+constexpr int kSmemBytes = 1024 + kOffX + kRows * 8;  // 1 KiB of alignment slack
 // Persistent mode needs the whole batch's units (sequence x KV head x pair of
 // query tiles) below this; the host launches one unit per cluster above it.
 constexpr int kMaxPersistentUnits = 16384;
@@ -114,9 +134,9 @@ constexpr int kSchedBins = 64;                      // work bins of the schedule
 static_assert(kThreads * kSchedBins * 2 + 4 * kSchedBins * 4 <= kVStages * kVStage, "schedule scratch");
 static_assert(kSmemBytes <= 227 * 1024, "shared memory");
 constexpr uint32_t kTmemCols = 512;
-// TMEM columns (the same in both CTAs): S buffers at 0 and 128, O at 256, two
-// P buffers (bf16 pairs packed in 32-bit columns, 64 columns each) at 384 and 448.
-constexpr uint32_t kColO = 256, kColP = 384;
+// TMEM columns (the same in both CTAs): S buffers at 0 and 128 (P, bf16 pairs
+// packed in 32-bit columns, over the first 64 of each), O_0 and O_1 at 256 and 384.
+constexpr uint32_t kColO = 256;
 constexpr float kRescaleLog2 = 8.0f;
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;
 
@@ -354,6 +374,39 @@ __device__ __forceinline__ bool wait_phase(uint32_t bar, uint32_t parity, volati
 __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int *abort, unsigned *status) {
     return __all_sync(0xffffffffu, wait_phase(bar, parity, abort, status));
 }
+// The waits of the producers and the softmax warps: the same bound, with a
+// suspend-time hint, so that a warp whose phase has not completed sleeps in
+// the barrier (woken when the phase completes, or after the hint) instead of
+// spinning on the issue slots of the SM sub-partition it shares with a
+// softmax warp that is computing.  The MMA issuer keeps spinning: its wake-up
+// latency lies on the tile's critical path.
+constexpr uint32_t kSuspendNs = 1000;
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity), "r"(kSuspendNs)
+        : "memory");
+    return ok != 0;
+}
+__device__ __forceinline__ bool wait_phase_sleep(uint32_t bar, uint32_t parity, volatile int *abort, unsigned *status) {
+    const unsigned long long t0 = global_ns();
+    while (!mbar_try_wait_sleep(bar, parity)) {
+        if (*abort) return false;
+        if (global_ns() - t0 > kWaitLimitNs) {
+            *abort = 1;
+            if (status) atomicOr(status, (unsigned)PS_DEVICE_TIMEOUT);
+            return false;
+        }
+    }
+    return true;
+}
+__device__ __forceinline__ bool warp_wait_sleep(uint32_t bar, uint32_t parity, volatile int *abort, unsigned *status) {
+    return __all_sync(0xffffffffu, wait_phase_sleep(bar, parity, abort, status));
+}
 // Bounded wait without the abort shortcut: used to drain this thread's own
 // copies and MMAs, which complete whatever the other roles did.
 __device__ __forceinline__ void drain_phase(uint32_t bar, uint32_t parity) {
@@ -500,7 +553,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     auto bar_vfree = [&](int st) { return saddr(bars + 2 + 2 * kKStages + kVStages + st); };
     constexpr int kB = 2 + 2 * kKStages + 2 * kVStages;
     auto bar_sfull = [&](int b) { return saddr(bars + kB + b); };
-    auto bar_sfree = [&](int b) { return saddr(bars + kB + 2 + b); };  // leader's
     auto bar_pfull = [&](int b) { return saddr(bars + kB + 4 + b); };  // leader's
     auto bar_pfree = [&](int b) { return saddr(bars + kB + 6 + b); };
     const uint32_t bar_mma_end = saddr(bars + kB + 8);
@@ -509,7 +561,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     volatile int *abort = reinterpret_cast<volatile int *>(bars + kB + 11);
     auto bar_qfree = [&](int qb) { return saddr(bars + kB + 12 + qb); };  // [2]
     const uint32_t bar_ofree = saddr(bars + kB + 14);                     // leader's
-    static_assert((2 + 2 * kKStages + 2 * kVStages + 15) * 8 <= kBarBytes, "barrier area");
+    auto bar_xfull = [&](int q) { return saddr(bars + kB + 16 + q); };   // [4] group 1 -> group 0, per lane quarter
+    auto bar_xempty = [&](int q) { return saddr(bars + kB + 20 + q); };  // [4]
+    static_assert((2 + 2 * kKStages + 2 * kVStages + 24) * 8 <= kBarBytes, "barrier area");
 
     if (tid == 0) {
         for (int i = 0; i < 2; ++i) {
@@ -526,13 +580,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(bar_sfull(i), 1);
-            mbar_init(bar_sfree(i), 8);  // four softmax warps in each CTA
-            mbar_init(bar_pfull(i), 8);
+            mbar_init(bar_pfull(i), 8);  // the buffer's four softmax warps in each CTA
             mbar_init(bar_pfree(i), 1);
         }
         mbar_init(bar_mma_end, 1);
         mbar_init(bar_vtail, 1);
-        mbar_init(bar_ofree, 8);  // both CTAs' softmax warps have read O
+        mbar_init(bar_ofree, 8);  // both CTAs' group 0 softmax warps have read O
+        for (int q = 0; q < 4; ++q) {
+            mbar_init(bar_xfull(q), 1);
+            mbar_init(bar_xempty(q), 1);
+        }
         *abort = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -553,7 +610,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     const uint32_t sQ = saddr(sm + kOffQ), sK = saddr(sm + kOffK), sV = saddr(sm + kOffV);
     bool bad_unused;
 
-    if (warp == 0 || warp == 6) {
+    if (warp < 4) {
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsCtl));
+    if (warp == 0 || warp == 2) {
         // ----------------------------------------------------- producers --
         const bool is_k = warp == 0;
         uint64_t keep;  // every K/V page is read by all query tiles of its (sequence, head)
@@ -572,7 +631,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             if (is_k) {
                 // Q of this unit into buffer ui & 1, once the Q K^T of unit ui - 2 is done.
                 const int qb = ui & 1;
-                if (ui >= 2 && !warp_wait(bar_qfree(qb), ((ui - 2) >> 1) & 1, abort, p.status)) { ok = false; break; }
+                if (ui >= 2 && !warp_wait_sleep(bar_qfree(qb), ((ui - 2) >> 1) & 1, abort, p.status)) { ok = false; break; }
                 if (lane == 0) {
                     const uint32_t lq = map_to(bar_q(qb), 0);
                     mbar_expect_tx_cluster(lq, (uint32_t)(2 * 128 * g * tpt));
@@ -585,7 +644,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             for (int n = 0; n < x.ntiles; ++n) {
                 const int st = issued % stages, use = issued / stages;
                 if (issued >= stages &&
-                    !warp_wait(is_k ? bar_kfree(st) : bar_vfree(st), (use - 1) & 1, abort, p.status)) { ok = false; break; }
+                    !warp_wait_sleep(is_k ? bar_kfree(st) : bar_vfree(st), (use - 1) & 1, abort, p.status)) { ok = false; break; }
                 const int base = n * kKeys;
                 if (is_k) {
                     // Keys 64 rank .. 64 rank + 63 of the tile, both 64-dim halves:
@@ -634,7 +693,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                         // rows past the needed keys (other tokens' data, or stale bytes)
                         // are zeroed -- P is zero there -- before the leader is told.
                         tail_pending = true;
-                        if (!warp_wait(bar_vtail, tails & 1, abort, p.status)) { ok = false; break; }
+                        if (!warp_wait_sleep(bar_vtail, tails & 1, abort, p.status)) { ok = false; break; }
                         tail_pending = false;
                         ++tails;
                         uint8_t *v = sm + kOffV + st * kVStage;
@@ -676,7 +735,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                     if (n < x.ntiles) {
                         const int t = t0 + n, st = t % kKStages, b = t & 1;
                         if (!warp_wait(bar_kfull(st), (t / kKStages) & 1, abort, p.status)) { ok = false; break; }
-                        if (t >= 2 && !warp_wait(bar_sfree(b), ((t >> 1) - 1) & 1, abort, p.status)) { ok = false; break; }
                         tc_fence_after();
                         if (lane == 0) {
                             const uint64_t kd = dK + (uint64_t)((st * kKStage) >> 4);
@@ -695,17 +753,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                         const int m = n - 1, t = t0 + m, st = t % kVStages;
                         if (!warp_wait(bar_vfull(st), (t / kVStages) & 1, abort, p.status)) { ok = false; break; }
                         if (!warp_wait(bar_pfull(t & 1), (t >> 1) & 1, abort, p.status)) { ok = false; break; }
-                        // The unit's first P V overwrites O: the previous unit's O must
-                        // have been read out by both CTAs' softmax warps.
+                        // The unit's first P V into each O buffer overwrites it: the
+                        // previous unit's O_0 and O_1 must have been read out by both
+                        // CTAs' group 0 softmax warps (the merge).
                         if (m == 0 && ui > 0 && !warp_wait(bar_ofree, (ui - 1) & 1, abort, p.status)) { ok = false; break; }
                         tc_fence_after();
                         if (lane == 0) {
-                            const uint32_t pt = tmem + kColP + (t & 1) * (kKeys / 2);
+                            const uint32_t pt = tmem + (t & 1) * kKeys;  // P over S
                             const uint64_t vd = dV + (uint64_t)((st * kVStage) >> 4);
 #pragma unroll
                             for (int kk = 0; kk < kKeys / 16; ++kk)
-                                umma2_ts(tmem + kColO, pt + kk * 8, vd + (uint64_t)((kk * (16 * 128)) >> 4), idO,
-                                         (m > 0 || kk > 0) ? 1u : 0u);
+                                umma2_ts(tmem + kColO + (t & 1) * kD, pt + kk * 8, vd + (uint64_t)((kk * (16 * 128)) >> 4), idO,
+                                         (m > 1 || kk > 0) ? 1u : 0u);
                             umma_commit_pair(bar_pfree(t & 1));
                             umma_commit_pair(bar_vfree(st));
                         }
@@ -720,13 +779,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             __syncwarp();
         }
         drain_phase(bar_mma_end, 0);
+    }
     } else {
+        asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegsSoftmax));
         // ------------------------------------------------------- softmax --
-        const int quarter = warp & 3;  // TMEM lanes 32 * quarter .. + 31
+        const int G = warp >= 8 ? 1 : 0;  // key tiles of global index = G (mod 2)
+        const int quarter = warp & 3;      // TMEM lanes 32 * quarter .. + 31
         const int r = quarter * 32 + lane;
         const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
         const int tl = r / g, hl = r - tl * g;
         const float sl2 = p.scale_log2;
+        float2 *xs = reinterpret_cast<float2 *>(sm + kOffX);
         bool ok = true;
         int t0 = 0;
         for (int ui = 0; ok && ui < nunits; ++ui) {
@@ -736,18 +799,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             const int limit = row_valid ? (x.L - x.Q + tok0 + tl + 1) : x.kv_limit;
             float m_ref = -INFINITY;
             uint64_t l2 = pack2(0.f, 0.f);  // row sum, as two interleaved partial sums
-            for (int n = 0; n < x.ntiles; ++n) {
-                const int t = t0 + n, b = t & 1;
-                if (!warp_wait(bar_sfull(b), (t >> 1) & 1, abort, p.status)) { ok = false; break; }
+            for (int n = ((t0 & 1) == G) ? 0 : 1; n < x.ntiles; n += 2) {
+                const int t = t0 + n;
+                if (!warp_wait_sleep(bar_sfull(G), (t >> 1) & 1, abort, p.status)) { ok = false; break; }
                 tc_fence_after();
                 float sv[kKeys];
 #pragma unroll
-                for (int c = 0; c < 4; ++c) tmem_ld32(trow + b * kKeys + c * 32, sv + c * 32);
+                for (int c = 0; c < 4; ++c) tmem_ld32(trow + G * kKeys + c * 32, sv + c * 32);
                 tmem_wait_ld();
                 tmem_loaded<kKeys>(sv);
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) mbar_arrive_cluster(map_to(bar_sfree(b), 0));
                 const int base = n * kKeys;
                 if (base + kKeys > limit) {
 #pragma unroll
@@ -759,21 +819,21 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                 for (int i = 1; i + 1 < kKeys; i += 2) mx = max3(mx, sv[i], sv[i + 1]);
                 mx = fmaxf(mx, sv[kKeys - 1]);
                 const float m_tile = mx * sl2;
-                const bool grow = m_tile > m_ref + kRescaleLog2;  // always true on a unit's first tile
+                const bool grow = m_tile > m_ref + kRescaleLog2;
                 const float alpha = grow ? ex2(m_ref - m_tile) : 1.f;
-                if (n >= 1 && __any_sync(0xffffffffu, grow)) {
-                    // O must hold key tiles 0 .. n-1 before it is rescaled.
-                    if (!warp_wait(bar_pfree((t - 1) & 1), ((t - 1) >> 1) & 1, abort, p.status)) { ok = false; break; }
+                if (n >= 2 && __any_sync(0xffffffffu, grow)) {
+                    // O_G must hold this group's earlier tiles before it is rescaled.
+                    if (!warp_wait_sleep(bar_pfree(G), ((t - 2) >> 1) & 1, abort, p.status)) { ok = false; break; }
                     tc_fence_after();
 #pragma unroll
                     for (int c = 0; c < 4; ++c) {
                         float ov[32];
-                        tmem_ld32(trow + kColO + c * 32, ov);
+                        tmem_ld32(trow + kColO + G * kD + c * 32, ov);
                         tmem_wait_ld();
                         tmem_loaded<32>(ov);
 #pragma unroll
                         for (int i = 0; i < 32; ++i) ov[i] *= alpha;
-                        tmem_st32(trow + kColO + c * 32, ov);
+                        tmem_st32(trow + kColO + G * kD + c * 32, ov);
                     }
                     tmem_wait_st();
                 }
@@ -781,14 +841,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                     l2 = mul2(l2, pack2(alpha, alpha));
                     m_ref = m_tile;
                 }
-                const uint64_t sl2x2 = pack2(sl2, sl2), nm2 = pack2(-m_ref, -m_ref);
-                // P buffer b was last read by the P V of tile t - 2.
-                if (t >= 2) {
-                    if (!warp_wait(bar_pfree(b), ((t >> 1) - 1) & 1, abort, p.status)) { ok = false; break; }
-                    tc_fence_after();
-                }
-                // P row (bf16 pairs) into TMEM buffer b, row = this thread's lane:
-                // the A operand of the P V MMA.
+                // A row whose keys in this group's tiles are all masked so far has
+                // m_ref = -inf: its weights are 0 (not inf - inf).
+                const float m_use = m_ref == -INFINITY ? 0.f : m_ref;
+                const uint64_t sl2x2 = pack2(sl2, sl2), nm2 = pack2(-m_use, -m_use);
+                // P (bf16 pairs) over the first 64 columns of this S buffer: the
+                // P V of tile t - 2, the last reader of those columns, finished
+                // before the Q K^T of tile t (whose completion was just waited for).
 #pragma unroll
                 for (int c = 0; c < 4; ++c) {
                     uint32_t w[16];
@@ -802,42 +861,71 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                         l2 = add2(l2, pack2(e0, e1));
                         w[e] = *reinterpret_cast<const uint32_t *>(&pr);
                     }
-                    tmem_st16u(trow + kColP + b * (kKeys / 2) + c * 16, w);
+                    tmem_st16u(trow + G * kKeys + c * 16, w);
                 }
                 tmem_wait_st();
                 tc_fence_before();
                 __syncwarp();
-                if (lane == 0) mbar_arrive_cluster(map_to(bar_pfull(b), 0));
+                if (lane == 0) mbar_arrive_cluster(map_to(bar_pfull(G), 0));
             }
             if (!ok) break;
-            const int tl_last = t0 + x.ntiles - 1;
-            if (!warp_wait(bar_pfree(tl_last & 1), (tl_last >> 1) & 1, abort, p.status)) { ok = false; break; }
-            tc_fence_after();
-            // O of this unit into registers, then the leader may start the next
-            // unit's P V (which overwrites O) while the rows are written out.
-            float ov[kD];
-#pragma unroll
-            for (int c = 0; c < 4; ++c) tmem_ld32(trow + kColO + c * 32, ov + c * 32);
-            tmem_wait_ld();
-            tmem_loaded<kD>(ov);
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive_cluster(map_to(bar_ofree, 0));
             float la, lb;
             unpack2(l2, la, lb);
-            const float inv = 1.f / (la + lb);
-            if (row_valid) {
-                uint16_t *orow = p.out + ((size_t)(x.qs0 + tok0 + tl) * p.num_q_heads + (size_t)x.j * g + hl) * kD;
+            if (G == 1) {
+                // Hand (m, l) of these rows to group 0, which merges the two halves.
+                if (ui > 0 && !warp_wait_sleep(bar_xempty(quarter), (ui - 1) & 1, abort, p.status)) { ok = false; break; }
+                xs[r] = make_float2(m_ref, la + lb);
+                __syncwarp();
+                if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar_xfull(quarter)) : "memory");
+            } else {
+                // Group 1's hand-off comes after its last softmax, so the barrier of
+                // the unit's last P V is then at most one phase behind: its parity
+                // wait cannot pass on an older phase.
+                if (!warp_wait_sleep(bar_xfull(quarter), ui & 1, abort, p.status)) { ok = false; break; }
+                const int tl_last = t0 + x.ntiles - 1;
+                if (!warp_wait_sleep(bar_pfree(tl_last & 1), (tl_last >> 1) & 1, abort, p.status)) { ok = false; break; }
+                const float2 o1 = xs[r];
+                __syncwarp();
+                if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar_xempty(quarter)) : "memory");
+                // Which buffers this unit's tiles used (a one-tile unit uses one).
+                const bool has0 = x.ntiles >= 2 || (t0 & 1) == 0, has1 = x.ntiles >= 2 || (t0 & 1) == 1;
+                const float m0 = m_ref, m1 = o1.x;
+                const float m = fmaxf(has0 ? m0 : -INFINITY, has1 ? m1 : -INFINITY);
+                const float c0 = has0 ? ex2(m0 - m) : 0.f, c1 = has1 ? ex2(m1 - m) : 0.f;
+                const float inv = 1.f / ((la + lb) * c0 + o1.y * c1);
+                const float f0 = c0 * inv, f1 = c1 * inv;
+                tc_fence_after();
+                // O = f0 O_0 + f1 O_1, 32 dims at a time, straight to the output
+                // row; then the leader may start the next unit's P V (which
+                // overwrites both accumulators).
+                uint16_t *orow = row_valid ? p.out + ((size_t)(x.qs0 + tok0 + tl) * p.num_q_heads + (size_t)x.j * g + hl) * kD : nullptr;
+#pragma unroll 1
+                for (int c = 0; c < 4; ++c) {
+                    // Both accumulators are read; one this unit left unused holds
+                    // stale values and is not used.
+                    float a0[32], a1[32];
+                    tmem_ld32(trow + kColO + c * 32, a0);
+                    tmem_ld32(trow + kColO + kD + c * 32, a1);
+                    tmem_wait_ld();
+                    tmem_loaded<32>(a0);
+                    tmem_loaded<32>(a1);
+                    uint32_t w[16];
 #pragma unroll
-                for (int v = 0; v < kD / 8; ++v) {
-                    uint32_t w[4];
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        const __nv_bfloat162 pr = __floats2bfloat162_rn(ov[v * 8 + 2 * e] * inv, ov[v * 8 + 2 * e + 1] * inv);
+                    for (int e = 0; e < 16; ++e) {
+                        float y0 = has0 ? a0[2 * e] * f0 : 0.f, y1 = has0 ? a0[2 * e + 1] * f0 : 0.f;
+                        y0 = has1 ? fmaf(a1[2 * e], f1, y0) : y0;
+                        y1 = has1 ? fmaf(a1[2 * e + 1], f1, y1) : y1;
+                        const __nv_bfloat162 pr = __floats2bfloat162_rn(y0, y1);
                         w[e] = *reinterpret_cast<const uint32_t *>(&pr);
                     }
-                    *reinterpret_cast<uint4 *>(orow + v * 8) = make_uint4(w[0], w[1], w[2], w[3]);
+                    if (row_valid)
+#pragma unroll
+                        for (int v = 0; v < 4; ++v)
+                            *reinterpret_cast<uint4 *>(orow + c * 32 + v * 8) = make_uint4(w[4 * v], w[4 * v + 1], w[4 * v + 2], w[4 * v + 3]);
                 }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive_cluster(map_to(bar_ofree, 0));
             }
             t0 += x.ntiles;
         }
@@ -925,6 +1013,9 @@ extern "C" ps_status_t ps_prefill_attention(const void *q, const void *k_cache, 
     if (cudaFuncSetAttribute(ps_prefill_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) !=
         cudaSuccess)
         return PS_ERR_CUDA;
+    cudaFuncAttributes fa;
+    if (cudaFuncGetAttributes(&fa, ps_prefill_kernel) != cudaSuccess) return PS_ERR_CUDA;
+    if (fa.numRegs * kThreads < 128 * kRegsCtl + 256 * kRegsSoftmax) return PS_ERR_UNSUPPORTED;
 
     PrefillParams pp;
     pp.block_table = block_table;

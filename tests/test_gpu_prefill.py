@@ -182,6 +182,35 @@ def test_full_size_prefill_every_row(psd):
     _compare(out, _oracle(wl), "p2, all %d outputs" % out.numel(), rel=0.0)
 
 
+def test_full_size_prefill_runs_are_bit_identical(psd):
+    """The kernel is deterministic (fixed tile order, fixed reduction order),
+    so repeated launches of the full-size batch give the same bits; a race
+    between the pipeline roles (a barrier wait passing on a stale phase, an
+    accumulator read before its last P V) shows up as runs that differ."""
+    wl = inputs.make_prefill_workload("p2", device="cuda")
+    first, status = _gpu(psd, wl)
+    assert status == 0
+    for i in range(12):
+        again, status = _gpu(psd, wl)
+        assert status == 0
+        assert torch.equal(again, first), "run %d differs from the first" % (i + 1)
+
+
+def test_prefill_short_units_persistent(psd):
+    """400 short chunks on short contexts (one to three 128-key tiles per
+    unit): persistent clusters whose units leave one softmax group with no
+    tile or a single one, every output against the oracle."""
+    rng = np.random.default_rng(41)
+    new = rng.integers(1, 65, size=400)
+    prior = rng.integers(0, 201, size=400)
+    wl = inputs.make_prefill_workload("p1", device="cpu", new=new, prior=prior, num_q_heads=32, num_kv_heads=8,
+                                      seed=41).to("cuda")
+    assert wl.seq_lens.shape[0] * 8 * ((wl.max_q_len + 31) // 32 + 1) // 2 <= 16384
+    out, status = _gpu(psd, wl)
+    assert status == 0
+    _compare(out, _oracle(wl), "400 short chunks")
+
+
 def test_prefill_with_more_units_than_a_persistent_launch_holds(psd):
     """Above 16384 units (sequence x KV head x pair of query tiles) the kernel
     runs one unit per cluster instead of persistent clusters: 2100 short
