@@ -354,6 +354,17 @@ __device__ __forceinline__ float ex2(float x) {
     return y;
 }
 
+__device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
 // Bounded wait; also returns false as soon as another role raised `abort`.
 __device__ __forceinline__ bool wait_phase(uint32_t bar, uint32_t parity, volatile int *abort, unsigned *status) {
     for (int i = 0; i < 64; ++i)
@@ -731,10 +742,20 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                 const int qb = ui & 1;
                 if (!warp_wait(bar_q(qb), (ui >> 1) & 1, abort, p.status)) { ok = false; break; }
                 const uint64_t dq = dQ + (uint64_t)((qb * kQBytes) >> 4);
+                // A barrier poll costs a shared-memory round trip while the tensor
+                // core streams operands: the next group's K or V barrier is tested
+                // before the current group's MMAs are issued (the result is used
+                // after them), and waited for only if it had not completed.
+                bool k_seen = false;
                 for (int n = 0; ok && n <= x.ntiles; ++n) {
+                    bool v_seen = false;
                     if (n < x.ntiles) {
                         const int t = t0 + n, st = t % kKStages, b = t & 1;
-                        if (!warp_wait(bar_kfull(st), (t / kKStages) & 1, abort, p.status)) { ok = false; break; }
+                        if (!__all_sync(0xffffffffu, k_seen) && !warp_wait(bar_kfull(st), (t / kKStages) & 1, abort, p.status)) { ok = false; break; }
+                        if (n >= 1) {
+                            const int tv = t - 1;
+                            v_seen = mbar_test(bar_vfull(tv % kVStages), (tv / kVStages) & 1);
+                        }
                         tc_fence_after();
                         if (lane == 0) {
                             const uint64_t kd = dK + (uint64_t)((st * kKStage) >> 4);
@@ -749,14 +770,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                         }
                         __syncwarp();
                     }
+                    k_seen = false;
                     if (n >= 1) {
                         const int m = n - 1, t = t0 + m, st = t % kVStages;
-                        if (!warp_wait(bar_vfull(st), (t / kVStages) & 1, abort, p.status)) { ok = false; break; }
+                        if (!__all_sync(0xffffffffu, v_seen) && !warp_wait(bar_vfull(st), (t / kVStages) & 1, abort, p.status)) { ok = false; break; }
                         if (!warp_wait(bar_pfull(t & 1), (t >> 1) & 1, abort, p.status)) { ok = false; break; }
                         // The unit's first P V into each O buffer overwrites it: the
                         // previous unit's O_0 and O_1 must have been read out by both
                         // CTAs' group 0 softmax warps (the merge).
                         if (m == 0 && ui > 0 && !warp_wait(bar_ofree, (ui - 1) & 1, abort, p.status)) { ok = false; break; }
+                        if (n < x.ntiles) {
+                            const int tk = t0 + n + 1;
+                            if (n + 1 < x.ntiles) k_seen = mbar_test(bar_kfull(tk % kKStages), (tk / kKStages) & 1);
+                        }
                         tc_fence_after();
                         if (lane == 0) {
                             const uint32_t pt = tmem + (t & 1) * kKeys;  // P over S
