@@ -609,18 +609,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     auto bar_vfull = [&](int st) { return saddr(bars + 2 + 2 * kKStages + st); };              // [kVStages], leader's
     auto bar_vfree = [&](int st) { return saddr(bars + 2 + 2 * kKStages + kVStages + st); };
     constexpr int kB = 2 + 2 * kKStages + 2 * kVStages;
-    auto bar_sfull = [&](int b) { return saddr(bars + kB + b); };
-    auto bar_pfull = [&](int b) { return saddr(bars + kB + 4 + b); };  // leader's
-    auto bar_pfree = [&](int b) { return saddr(bars + kB + 6 + b); };
-    const uint32_t bar_mma_end = saddr(bars + kB + 8);
-    const uint32_t bar_vtail = saddr(bars + kB + 9);
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + kB + 10);
-    volatile int *abort = reinterpret_cast<volatile int *>(bars + kB + 11);
-    auto bar_qfree = [&](int qb) { return saddr(bars + kB + 12 + qb); };  // [2]
-    const uint32_t bar_ofree = saddr(bars + kB + 14);                     // leader's
-    auto bar_xfull = [&](int q) { return saddr(bars + kB + 16 + q); };   // [4] group 1 -> group 0, per lane quarter
-    auto bar_xempty = [&](int q) { return saddr(bars + kB + 20 + q); };  // [4]
-    static_assert((2 + 2 * kKStages + 2 * kVStages + 24) * 8 <= kBarBytes, "barrier area");
+    auto bar_sfull = [&](int b) { return saddr(bars + kB + b); };      // [2]
+    auto bar_pfull = [&](int b) { return saddr(bars + kB + 2 + b); };  // [2] leader's
+    auto bar_pfree = [&](int b) { return saddr(bars + kB + 4 + b); };  // [2]
+    const uint32_t bar_mma_end = saddr(bars + kB + 6);
+    const uint32_t bar_vtail = saddr(bars + kB + 7);
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + kB + 8);
+    volatile int *abort = reinterpret_cast<volatile int *>(bars + kB + 9);
+    auto bar_qfree = [&](int qb) { return saddr(bars + kB + 10 + qb); };  // [2]
+    const uint32_t bar_ofree = saddr(bars + kB + 12);                     // leader's
+    auto bar_xfull = [&](int q) { return saddr(bars + kB + 13 + q); };   // [4] group 1 -> group 0, per lane quarter
+    auto bar_xempty = [&](int q) { return saddr(bars + kB + 17 + q); };  // [4]
+    static_assert((2 + 2 * kKStages + 2 * kVStages + 21) * 8 <= kBarBytes, "barrier area");
 
     if (tid == 0) {
         for (int i = 0; i < 2; ++i) {
@@ -825,9 +825,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                         // previous unit's O_0 and O_1 must have been read out by both
                         // CTAs' group 0 softmax warps (the merge).
                         if (m == 0 && ui > 0 && !warp_wait(bar_ofree, (ui - 1) & 1, abort, p.status)) { ok = false; break; }
-                        if (n < x.ntiles) {
+                        if (n + 1 < x.ntiles) {
                             const int tk = t0 + n + 1;
-                            if (n + 1 < x.ntiles) k_seen = mbar_test(bar_kfull(tk % kKStages), (tk / kKStages) & 1);
+                            k_seen = mbar_test(bar_kfull(tk % kKStages), (tk / kKStages) & 1);
                         }
                         tc_fence_after();
                         if (lane == 0) {
