@@ -150,6 +150,7 @@ void ps::note_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 namespace {
 std::atomic<int> g_inject_launch_error{0};
 std::atomic<long long> g_inject_stall_ns{0};
+std::atomic<long long> g_inject_prefill_stall_ns{0};
 }  // namespace
 
 cudaError_t ps::take_injected_launch_error() {
@@ -157,6 +158,10 @@ cudaError_t ps::take_injected_launch_error() {
 }
 
 long long ps::take_injected_stall_ns() { return g_inject_stall_ns.exchange(0, std::memory_order_acq_rel); }
+
+long long ps::take_injected_prefill_stall_ns() {
+    return g_inject_prefill_stall_ns.exchange(0, std::memory_order_acq_rel);
+}
 
 ps_status_t ps_test_inject(int kind, long long value) {
     switch (kind) {
@@ -167,6 +172,10 @@ ps_status_t ps_test_inject(int kind, long long value) {
         case PS_INJECT_DECODE_STALL:
             if (value != 0 && (value < 1000 || value > 1000000000)) return PS_ERR_INVALID_ARG;
             g_inject_stall_ns.store(value, std::memory_order_release);
+            return PS_OK;
+        case PS_INJECT_PREFILL_STALL:
+            if (value != 0 && (value < 1000 || value > 1000000000)) return PS_ERR_INVALID_ARG;
+            g_inject_prefill_stall_ns.store(value, std::memory_order_release);
             return PS_OK;
         default:
             return PS_ERR_INVALID_ARG;

@@ -138,9 +138,11 @@ void note_launch();
 
 // One-shot faults set by ps_test_inject(): the CUDA error the next launch
 // reports instead of launching (cudaSuccess: none), and the stall the next
-// decode launch makes (0: none).  Each call consumes what it returns.
+// decode or prefill launch makes (0: none).  Each call consumes what it
+// returns.
 cudaError_t take_injected_launch_error();
 long long take_injected_stall_ns();
+long long take_injected_prefill_stall_ns();
 
 cudaError_t launch_decode(const DecodeParams &p, const CUtensorMap &tmK, const CUtensorMap &tmV, int grid_ctas,
                           size_t smem_bytes, cudaStream_t stream);

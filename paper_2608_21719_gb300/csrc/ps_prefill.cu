@@ -150,6 +150,7 @@ struct PrefillParams {
     float scale_log2;
     int persistent;    // 1: grid of clusters, each running a list of units; 0: one unit per cluster
     int num_clusters;  // persistent mode: clusters in the grid
+    long long test_stall_ns;  // > 0: injected stall (ps_test_inject), else 0
 };
 
 // ------------------------------------------------------------ PTX wrappers --
@@ -411,16 +412,25 @@ __device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity) {
         : "memory");
     return ok != 0;
 }
+// A wait ran out: every role of this CTA and of the other CTA of the pair
+// stops waiting at its next poll (both CTAs' abort flags are raised), and the
+// status word records the timeout.
+__device__ __forceinline__ void raise_abort(volatile int *abort, unsigned *status) {
+    *abort = 1;
+    const uint32_t peer = map_to(saddr(const_cast<int *>(abort)), cta_rank() ^ 1u);
+    asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(peer), "r"(1) : "memory");
+    if (status) atomicOr(status, (unsigned)PS_DEVICE_TIMEOUT);
+}
 // Bounded wait; also returns false as soon as another role raised `abort`.
-__device__ __forceinline__ bool wait_phase(uint32_t bar, uint32_t parity, volatile int *abort, unsigned *status) {
+__device__ __forceinline__ bool wait_phase(uint32_t bar, uint32_t parity, volatile int *abort, unsigned *status,
+                                           unsigned long long limit_ns = kWaitLimitNs) {
     for (int i = 0; i < 64; ++i)
         if (mbar_try_wait(bar, parity)) return true;
     const unsigned long long t0 = global_ns();
     while (!mbar_try_wait(bar, parity)) {
         if (*abort) return false;
-        if (global_ns() - t0 > kWaitLimitNs) {
-            *abort = 1;
-            if (status) atomicOr(status, (unsigned)PS_DEVICE_TIMEOUT);
+        if (global_ns() - t0 > limit_ns) {
+            raise_abort(abort, status);
             return false;
         }
     }
@@ -428,8 +438,9 @@ __device__ __forceinline__ bool wait_phase(uint32_t bar, uint32_t parity, volati
 }
 // The same, taken by a whole warp: every lane waits and the warp agrees on
 // the outcome, so the warp stays converged for .sync.aligned instructions.
-__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int *abort, unsigned *status) {
-    return __all_sync(0xffffffffu, wait_phase(bar, parity, abort, status));
+__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int *abort, unsigned *status,
+                                          unsigned long long limit_ns = kWaitLimitNs) {
+    return __all_sync(0xffffffffu, wait_phase(bar, parity, abort, status, limit_ns));
 }
 // The waits of the producers and the softmax warps: the same bound, with a
 // suspend-time hint, so that a warp whose phase has not completed sleeps in
@@ -454,8 +465,7 @@ __device__ __forceinline__ bool wait_phase_sleep(uint32_t bar, uint32_t parity, 
     while (!mbar_try_wait_sleep(bar, parity)) {
         if (*abort) return false;
         if (global_ns() - t0 > kWaitLimitNs) {
-            *abort = 1;
-            if (status) atomicOr(status, (unsigned)PS_DEVICE_TIMEOUT);
+            raise_abort(abort, status);
             return false;
         }
     }
@@ -620,7 +630,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     const uint32_t bar_ofree = saddr(bars + kB + 12);                     // leader's
     auto bar_xfull = [&](int q) { return saddr(bars + kB + 13 + q); };   // [4] group 1 -> group 0, per lane quarter
     auto bar_xempty = [&](int q) { return saddr(bars + kB + 17 + q); };  // [4]
-    static_assert((2 + 2 * kKStages + 2 * kVStages + 21) * 8 <= kBarBytes, "barrier area");
+    const uint32_t bar_stall = saddr(bars + kB + 21);  // nothing arrives on it: the injected stall (tests only)
+    static_assert((2 + 2 * kKStages + 2 * kVStages + 22) * 8 <= kBarBytes, "barrier area");
 
     if (tid == 0) {
         for (int i = 0; i < 2; ++i) {
@@ -643,6 +654,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         mbar_init(bar_mma_end, 1);
         mbar_init(bar_vtail, 1);
         mbar_init(bar_ofree, 8);  // both CTAs' group 0 softmax warps have read O
+        mbar_init(bar_stall, 1);
         for (int q = 0; q < 4; ++q) {
             mbar_init(bar_xfull(q), 1);
             mbar_init(bar_xempty(q), 1);
@@ -782,6 +794,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             // 14-bit start-address field (shared-memory addresses stay below 256 KiB).
             const uint64_t dQ = smem_desc(sQ, 16, 1024), dK = smem_desc(sK, 16, 1024), dV = smem_desc(sV, 16, 1024);
             bool ok = true;
+            // Injected stall (tests only): a wait that runs out before the first
+            // MMA, taking the same path as a real one.
+            if (p.test_stall_ns > 0 && !warp_wait(bar_stall, 0u, abort, p.status, (unsigned long long)p.test_stall_ns))
+                ok = false;
             int t0 = 0;  // tiles of the earlier units (S/P buffers and K/V stages run on across units)
             for (int ui = 0; ok && ui < nunits; ++ui) {
                 const Unit x = unit_of(p, ulist[ui], npairs, bad_unused);
@@ -1117,6 +1133,7 @@ extern "C" ps_status_t ps_prefill_attention(const void *q, const void *k_cache, 
     const int clusters = max(1, sms / 2);
     pp.persistent = (units <= kMaxPersistentUnits && (units + clusters - 1) / clusters <= kMaxUnitsPerCluster) ? 1 : 0;
     pp.num_clusters = clusters;
+    pp.test_stall_ns = ps::take_injected_prefill_stall_ns();
     const dim3 grid = pp.persistent ? dim3((unsigned)(2 * clusters), 1, 1)
                                     : dim3((unsigned)(2 * npairs), (unsigned)num_kv_heads, (unsigned)num_seqs);
     if (ps::take_injected_launch_error() != cudaSuccess) return PS_ERR_CUDA;

@@ -37,6 +37,7 @@ PS_DEVICE_BAD_BLOCK = 2
 PS_DEVICE_LEN_CLAMPED = 4
 PS_INJECT_LAUNCH_ERROR = 1
 PS_INJECT_DECODE_STALL = 2
+PS_INJECT_PREFILL_STALL = 3
 PS_NOALLOC_SCRATCH_BYTES = 16 << 20  # size of the workspace-free entry point's fixed device array
 
 

@@ -212,8 +212,9 @@ def test_kv_transfer_validates_on_the_host():
 
 
 def test_fault_injection_arguments():
-    for kind, value in [(0, 1), (3, 1), (psd.PS_INJECT_LAUNCH_ERROR, -1), (psd.PS_INJECT_LAUNCH_ERROR, 10001),
-                        (psd.PS_INJECT_DECODE_STALL, 999), (psd.PS_INJECT_DECODE_STALL, 2 * 10**9)]:
+    for kind, value in [(0, 1), (4, 1), (psd.PS_INJECT_LAUNCH_ERROR, -1), (psd.PS_INJECT_LAUNCH_ERROR, 10001),
+                        (psd.PS_INJECT_DECODE_STALL, 999), (psd.PS_INJECT_DECODE_STALL, 2 * 10**9),
+                        (psd.PS_INJECT_PREFILL_STALL, 999), (psd.PS_INJECT_PREFILL_STALL, 2 * 10**9)]:
         with pytest.raises(psd.PsError) as ei:
             psd.ps_test_inject(kind, value)
         assert ei.value.status == psd.PS_ERR_INVALID_ARG
@@ -222,3 +223,5 @@ def test_fault_injection_arguments():
     psd.ps_test_inject(psd.PS_INJECT_LAUNCH_ERROR, 0)
     psd.ps_test_inject(psd.PS_INJECT_DECODE_STALL, 10**6)
     psd.ps_test_inject(psd.PS_INJECT_DECODE_STALL, 0)
+    psd.ps_test_inject(psd.PS_INJECT_PREFILL_STALL, 10**6)
+    psd.ps_test_inject(psd.PS_INJECT_PREFILL_STALL, 0)

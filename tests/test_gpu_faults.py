@@ -28,6 +28,7 @@ def psd():
     yield ps_decode
     ps_decode.ps_test_inject(ps_decode.PS_INJECT_LAUNCH_ERROR, 0)
     ps_decode.ps_test_inject(ps_decode.PS_INJECT_DECODE_STALL, 0)
+    ps_decode.ps_test_inject(ps_decode.PS_INJECT_PREFILL_STALL, 0)
 
 
 def _oracle(wl):
@@ -59,6 +60,48 @@ def test_injected_launch_error_is_reported_and_the_next_call_works(psd):
     assert attn.device_status() == 0
     _check(out, _oracle(wl))
     attn.close()
+
+
+@pytest.mark.parametrize("persistent", [True, False])
+def test_injected_prefill_stall_times_out_and_the_next_call_works(psd, persistent):
+    """The MMA issuer of every CTA pair first waits 2 ms on an mbarrier that
+    nothing arrives on: the wait runs out, both CTAs of every pair give up
+    (each raises the other's abort flag), PS_DEVICE_TIMEOUT is set, the copies
+    in flight land, tensor memory is freed and no output is written; the next
+    call on the same context is normal and matches the oracle.  Both launch
+    forms: persistent clusters, and one unit per cluster (above 16384 units)."""
+    if persistent:
+        wl = inputs.make_prefill_workload("p1", device="cpu", new=[300, 90, 1], prior=[500, 0, 40],
+                                          num_q_heads=32, num_kv_heads=8, seed=5)
+    else:
+        rng = np.random.default_rng(31)
+        wl = inputs.make_prefill_workload("p1", device="cpu", new=rng.integers(1, 33, size=2100),
+                                          prior=rng.integers(0, 60, size=2100), num_q_heads=32, num_kv_heads=8,
+                                          seed=31)
+    wl = wl.to("cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    sentinel = torch.full_like(wl.q, 3.0)
+    psd.ps_test_inject(psd.PS_INJECT_PREFILL_STALL, 2_000_000)
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    start.record()
+    out = psd.prefill_attention(wl.q, wl.k_cache, wl.v_cache, wl.block_table, wl.seq_lens, wl.q_start,
+                                wl.max_q_len, out=sentinel.clone(), scale=wl.scale, device_status=status)
+    end.record()
+    torch.cuda.synchronize()
+    ms = start.elapsed_time(end)
+    assert 1.9 <= ms < 1000.0, ms  # ran to the injected limit; the other waits gave up with it
+    assert int(status.item()) & psd.PS_DEVICE_TIMEOUT
+    assert torch.equal(out, sentinel)  # no MMA ran, so no row was written
+    status.zero_()
+    out = psd.prefill_attention(wl.q, wl.k_cache, wl.v_cache, wl.block_table, wl.seq_lens, wl.q_start,
+                                wl.max_q_len, scale=wl.scale, device_status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    ref = oracle.prefill_attention(inputs.bf16_bits(wl.q), inputs.bf16_bits(wl.k_cache),
+                                   inputs.bf16_bits(wl.v_cache), wl.block_table.cpu().numpy(), wl.lengths,
+                                   wl.q_start.cpu().numpy(), wl.k_cache.shape[1], wl.scale)
+    err = np.abs(out.float().cpu().numpy().astype(np.float64) - ref)
+    assert err.max() <= MAX_ABS + 2.0 ** -8 * np.abs(ref).max() and err.mean() <= MEAN_ABS, (err.max(), err.mean())
 
 
 def test_injected_launch_error_on_prefill_and_kv_pack(psd):
