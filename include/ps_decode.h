@@ -347,10 +347,10 @@ ps_status_t ps_decode_attention_noalloc(const void *q, const void *k_cache, cons
  *                           the copies it has in flight land and exits
  *                           without writing any output (which is then
  *                           invalid).  Recovery is the documented one.
- *   PS_INJECT_PREFILL_STALL the next chunked-prefill launch makes the MMA
- *                           issuer of every CTA pair first wait, for `value`
- *                           ns (1000 .. 1000000000), on an mbarrier that
- *                           nothing arrives on.  The wait runs out as a real
+ *   PS_INJECT_PREFILL_STALL the next chunked-prefill launch makes one
+ *                           softmax warpgroup of every CTA pair first wait,
+ *                           for `value` ns (1000 .. 1000000000), on an
+ *                           mbarrier that nothing arrives on.  The wait runs out as a real
  *                           stall would: both CTAs of every pair give up,
  *                           PS_DEVICE_TIMEOUT is raised, the copies in flight
  *                           land, tensor memory is freed and the kernel exits

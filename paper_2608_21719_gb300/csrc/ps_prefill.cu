@@ -412,25 +412,27 @@ __device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity) {
         : "memory");
     return ok != 0;
 }
-// A wait ran out: every role of this CTA and of the other CTA of the pair
-// stops waiting at its next poll (both CTAs' abort flags are raised), and the
-// status word records the timeout.
-__device__ __forceinline__ void raise_abort(volatile int *abort, unsigned *status) {
-    *abort = 1;
+// The softmax warps of a CTA that gave up (one of its waits ran out, here or
+// in another role of the CTA) raise the abort flag of the other CTA of the
+// pair too, so that every role there stops waiting at its next poll instead
+// of at its own limit: every role of a CTA that gives up ends its loops, the
+// softmax warps included.  Called once, where the softmax warps leave their
+// loops: kept out of the waits and the control warps, whose code it would
+// otherwise enlarge on the hot path.
+__device__ __noinline__ void raise_peer_abort(volatile int *abort) {
     const uint32_t peer = map_to(saddr(const_cast<int *>(abort)), cta_rank() ^ 1u);
     asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(peer), "r"(1) : "memory");
-    if (status) atomicOr(status, (unsigned)PS_DEVICE_TIMEOUT);
 }
 // Bounded wait; also returns false as soon as another role raised `abort`.
-__device__ __forceinline__ bool wait_phase(uint32_t bar, uint32_t parity, volatile int *abort, unsigned *status,
-                                           unsigned long long limit_ns = kWaitLimitNs) {
+__device__ __forceinline__ bool wait_phase(uint32_t bar, uint32_t parity, volatile int *abort, unsigned *status) {
     for (int i = 0; i < 64; ++i)
         if (mbar_try_wait(bar, parity)) return true;
     const unsigned long long t0 = global_ns();
     while (!mbar_try_wait(bar, parity)) {
         if (*abort) return false;
-        if (global_ns() - t0 > limit_ns) {
-            raise_abort(abort, status);
+        if (global_ns() - t0 > kWaitLimitNs) {
+            *abort = 1;
+            if (status) atomicOr(status, (unsigned)PS_DEVICE_TIMEOUT);
             return false;
         }
     }
@@ -438,9 +440,24 @@ __device__ __forceinline__ bool wait_phase(uint32_t bar, uint32_t parity, volati
 }
 // The same, taken by a whole warp: every lane waits and the warp agrees on
 // the outcome, so the warp stays converged for .sync.aligned instructions.
-__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int *abort, unsigned *status,
-                                          unsigned long long limit_ns = kWaitLimitNs) {
-    return __all_sync(0xffffffffu, wait_phase(bar, parity, abort, status, limit_ns));
+__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int *abort, unsigned *status) {
+    return __all_sync(0xffffffffu, wait_phase(bar, parity, abort, status));
+}
+// The injected stall (tests only): a wait with the given limit on a barrier
+// that nothing arrives on, giving up the way every wait does.
+__device__ __forceinline__ bool stall_wait(uint32_t bar, unsigned long long limit_ns, volatile int *abort, unsigned *status) {
+    const unsigned long long t0 = global_ns();
+    bool ok = true;
+    while (!mbar_try_wait(bar, 0u)) {
+        if (*abort) { ok = false; break; }
+        if (global_ns() - t0 > limit_ns) {
+            *abort = 1;
+            if (status) atomicOr(status, (unsigned)PS_DEVICE_TIMEOUT);
+            ok = false;
+            break;
+        }
+    }
+    return __all_sync(0xffffffffu, ok);
 }
 // The waits of the producers and the softmax warps: the same bound, with a
 // suspend-time hint, so that a warp whose phase has not completed sleeps in
@@ -465,7 +482,8 @@ __device__ __forceinline__ bool wait_phase_sleep(uint32_t bar, uint32_t parity, 
     while (!mbar_try_wait_sleep(bar, parity)) {
         if (*abort) return false;
         if (global_ns() - t0 > kWaitLimitNs) {
-            raise_abort(abort, status);
+            *abort = 1;
+            if (status) atomicOr(status, (unsigned)PS_DEVICE_TIMEOUT);
             return false;
         }
     }
@@ -794,10 +812,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             // 14-bit start-address field (shared-memory addresses stay below 256 KiB).
             const uint64_t dQ = smem_desc(sQ, 16, 1024), dK = smem_desc(sK, 16, 1024), dV = smem_desc(sV, 16, 1024);
             bool ok = true;
-            // Injected stall (tests only): a wait that runs out before the first
-            // MMA, taking the same path as a real one.
-            if (p.test_stall_ns > 0 && !warp_wait(bar_stall, 0u, abort, p.status, (unsigned long long)p.test_stall_ns))
-                ok = false;
             int t0 = 0;  // tiles of the earlier units (S/P buffers and K/V stages run on across units)
             for (int ui = 0; ok && ui < nunits; ++ui) {
                 const Unit x = unit_of(p, ulist[ui], npairs, bad_unused);
@@ -879,6 +893,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         const float sl2 = p.scale_log2;
         float2 *xs = reinterpret_cast<float2 *>(sm + kOffX);
         bool ok = true;
+        // Injected stall (tests only): group 0 of the leader CTA waits, before
+        // its first score tile, on a barrier nothing arrives on, so the
+        // leader's first P V never issues and the wait runs out the way a
+        // real one would.
+        if (p.test_stall_ns > 0 && G == 0 && rank == 0 &&
+            !stall_wait(bar_stall, (unsigned long long)p.test_stall_ns, abort, p.status))
+            ok = false;
         int t0 = 0;
         for (int ui = 0; ok && ui < nunits; ++ui) {
             const Unit x = unit_of(p, ulist[ui], npairs, bad_unused);
@@ -1017,6 +1038,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             }
             t0 += x.ntiles;
         }
+        if (!ok && lane == 0) raise_peer_abort(abort);
     }
     // Neither CTA leaves (nor frees TMEM) while the other may still touch its
     // shared memory or the leader's MMAs may still run.
