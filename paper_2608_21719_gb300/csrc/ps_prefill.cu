@@ -36,7 +36,11 @@
 //              buffer n & 1 of both CTAs (M = 256, N = 128, K = 128), and, once
 //              both CTAs' softmax has written P_n, O_{n & 1} += P_n V_n with P
 //              read from TMEM; tcgen05.commit multicasts each completion to
-//              both CTAs' barriers.
+//              both CTAs' barriers.  A tile's K and V copies (both CTAs')
+//              complete on one barrier, and the one commit after its P V
+//              frees both stages: each commit and each barrier poll is issuer
+//              time during which the tensor pipe runs dry, so the issuer keeps
+//              one poll and two commits (S full, K/V free) per tile.
 //   warp 3     idle (completes warpgroup 0).
 //   warps 4-7  softmax group 0: the tiles of even global index n;
 //   warps 8-11 softmax group 1: the tiles of odd n.  One TMEM lane (= one
@@ -97,14 +101,12 @@ constexpr int kD = 128;            // head_dim
 constexpr int kRows = 128;         // query rows per CTA (MMA M = 256 over the pair)
 constexpr int kKeys = 128;         // MMA N of S, K of P.V: keys per tile
 constexpr int kChunk = 16;         // keys per TMA box (one page slice)
-#ifndef PS_PREFILL_KSTAGES
-#define PS_PREFILL_KSTAGES 4
+#ifndef PS_PREFILL_STAGES
+#define PS_PREFILL_STAGES 4
 #endif
-#ifndef PS_PREFILL_VSTAGES
-#define PS_PREFILL_VSTAGES 4
-#endif
-constexpr int kKStages = PS_PREFILL_KSTAGES;  // K ring: a stage is free once its Q K^T is done
-constexpr int kVStages = PS_PREFILL_VSTAGES;  // V ring: a stage is free once its P V is done
+// K and V rings of the same depth: a tile's K and V land on one barrier and
+// their stages are freed together, once the tile's P V is done.
+constexpr int kStages = PS_PREFILL_STAGES;
 constexpr int kThreads = 384;
 // Registers per thread after the role split: warpgroup 0 (producers, MMA
 // issuer) gives registers back, the two softmax warpgroups take them.  The sum
@@ -120,8 +122,8 @@ constexpr int kKStage = 2 * kKHalf;           // 16 KiB
 constexpr int kVStage = kKeys * 128;          // 128 keys x this CTA's 64 dims: 16 KiB
 constexpr int kOffQ = 0;                            // two Q buffers: the next unit's Q loads early
 constexpr int kOffK = kOffQ + 2 * kQBytes;
-constexpr int kOffV = kOffK + kKStages * kKStage;
-constexpr int kOffBar = kOffV + kVStages * kVStage;
+constexpr int kOffV = kOffK + kStages * kKStage;
+constexpr int kOffBar = kOffV + kStages * kVStage;
 constexpr int kBarBytes = 512;
 constexpr int kMaxUnitsPerCluster = 256;            // a cluster's unit list (persistent mode)
 constexpr int kOffList = kOffBar + kBarBytes;
@@ -131,7 +133,7 @@ constexpr int kSmemBytes = 1024 + kOffX + kRows * 8;  // 1 KiB of alignment slac
 // query tiles) below this; the host launches one unit per cluster above it.
 constexpr int kMaxPersistentUnits = 16384;
 constexpr int kSchedBins = 64;                      // work bins of the schedule's counting sort
-static_assert(kThreads * kSchedBins * 2 + 4 * kSchedBins * 4 <= kVStages * kVStage, "schedule scratch");
+static_assert(kThreads * kSchedBins * 2 + 4 * kSchedBins * 4 <= kStages * kVStage, "schedule scratch");
 static_assert(kSmemBytes <= 227 * 1024, "shared memory");
 constexpr uint32_t kTmemCols = 512;
 // TMEM columns (the same in both CTAs): S buffers at 0 and 128 (P, bf16 pairs
@@ -632,42 +634,36 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 
     uint64_t *bars = reinterpret_cast<uint64_t *>(sm + kOffBar);
     auto bar_q = [&](int qb) { return saddr(bars + qb); };                                    // [2] leader's
-    auto bar_kfull = [&](int st) { return saddr(bars + 2 + st); };                             // [kKStages], leader's
-    auto bar_kfree = [&](int st) { return saddr(bars + 2 + kKStages + st); };                  // [kKStages]
-    auto bar_vfull = [&](int st) { return saddr(bars + 2 + 2 * kKStages + st); };              // [kVStages], leader's
-    auto bar_vfree = [&](int st) { return saddr(bars + 2 + 2 * kKStages + kVStages + st); };
-    constexpr int kB = 2 + 2 * kKStages + 2 * kVStages;
+    // K and V tile t: both CTAs' K and V copies complete on kvfull(t % kStages)
+    // (the leader's); the tile's P V commit frees both stages through kvfree.
+    auto bar_kvfull = [&](int st) { return saddr(bars + 2 + st); };           // [kStages], leader's
+    auto bar_kvfree = [&](int st) { return saddr(bars + 2 + kStages + st); };  // [kStages]
+    constexpr int kB = 2 + 2 * kStages;
     auto bar_sfull = [&](int b) { return saddr(bars + kB + b); };      // [2]
     auto bar_pfull = [&](int b) { return saddr(bars + kB + 2 + b); };  // [2] leader's
-    auto bar_pfree = [&](int b) { return saddr(bars + kB + 4 + b); };  // [2]
-    const uint32_t bar_mma_end = saddr(bars + kB + 6);
-    const uint32_t bar_vtail = saddr(bars + kB + 7);
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + kB + 8);
-    volatile int *abort = reinterpret_cast<volatile int *>(bars + kB + 9);
-    auto bar_qfree = [&](int qb) { return saddr(bars + kB + 10 + qb); };  // [2]
-    const uint32_t bar_ofree = saddr(bars + kB + 12);                     // leader's
-    auto bar_xfull = [&](int q) { return saddr(bars + kB + 13 + q); };   // [4] group 1 -> group 0, per lane quarter
-    auto bar_xempty = [&](int q) { return saddr(bars + kB + 17 + q); };  // [4]
-    const uint32_t bar_stall = saddr(bars + kB + 21);  // nothing arrives on it: the injected stall (tests only)
-    static_assert((2 + 2 * kKStages + 2 * kVStages + 22) * 8 <= kBarBytes, "barrier area");
+    const uint32_t bar_mma_end = saddr(bars + kB + 4);
+    const uint32_t bar_vtail = saddr(bars + kB + 5);
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + kB + 6);
+    volatile int *abort = reinterpret_cast<volatile int *>(bars + kB + 7);
+    auto bar_qfree = [&](int qb) { return saddr(bars + kB + 8 + qb); };  // [2]
+    const uint32_t bar_ofree = saddr(bars + kB + 10);                    // leader's
+    auto bar_xfull = [&](int q) { return saddr(bars + kB + 11 + q); };   // [4] group 1 -> group 0, per lane quarter
+    auto bar_xempty = [&](int q) { return saddr(bars + kB + 15 + q); };  // [4]
+    const uint32_t bar_stall = saddr(bars + kB + 19);  // nothing arrives on it: the injected stall (tests only)
+    static_assert((2 + 2 * kStages + 20) * 8 <= kBarBytes, "barrier area");
 
     if (tid == 0) {
         for (int i = 0; i < 2; ++i) {
             mbar_init(bar_q(i), 2);  // one arrival (with its bytes) from each CTA
             mbar_init(bar_qfree(i), 1);
         }
-        for (int i = 0; i < kKStages; ++i) {
-            mbar_init(bar_kfull(i), 2);
-            mbar_init(bar_kfree(i), 1);
-        }
-        for (int i = 0; i < kVStages; ++i) {
-            mbar_init(bar_vfull(i), 2);
-            mbar_init(bar_vfree(i), 1);
+        for (int i = 0; i < kStages; ++i) {
+            mbar_init(bar_kvfull(i), 4);  // the K and the V arrival (with its bytes) of each CTA
+            mbar_init(bar_kvfree(i), 1);
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(bar_sfull(i), 1);
             mbar_init(bar_pfull(i), 8);  // the buffer's four softmax warps in each CTA
-            mbar_init(bar_pfree(i), 1);
         }
         mbar_init(bar_mma_end, 1);
         mbar_init(bar_vtail, 1);
@@ -708,7 +704,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(is_k ? &tmK : &tmV)) : "memory");
             if (is_k) asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmQ)) : "memory");
         }
-        const int stages = is_k ? kKStages : kVStages;
+        constexpr int stages = kStages;
         int issued = 0, tails = 0, units_q = 0;
         bool tail_pending = false, ok = true;
         for (int ui = 0; ok && ui < nunits; ++ui) {
@@ -731,14 +727,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             for (int n = 0; n < x.ntiles; ++n) {
                 const int st = issued % stages, use = issued / stages;
                 if (issued >= stages &&
-                    !warp_wait_sleep(is_k ? bar_kfree(st) : bar_vfree(st), (use - 1) & 1, abort, p.status)) { ok = false; break; }
+                    !warp_wait_sleep(bar_kvfree(st), (use - 1) & 1, abort, p.status)) { ok = false; break; }
                 const int base = n * kKeys;
                 if (is_k) {
                     // Keys 64 rank .. 64 rank + 63 of the tile, both 64-dim halves:
                     // lanes 0-7 take (chunk lane & 3, half lane >> 2).
                     const int k0 = base + kPairKeys * (int)rank;
                     const int nc = max(0, min(kPairKeys / kChunk, (x.kv_limit - k0 + kChunk - 1) / kChunk));
-                    const uint32_t full = map_to(bar_kfull(st), 0);
+                    const uint32_t full = map_to(bar_kvfull(st), 0);
                     if (lane == 0) mbar_expect_tx_cluster(full, (uint32_t)(nc * 2 * kChunk * 128));
                     __syncwarp();
                     const int c = lane & 3, half = lane >> 2;
@@ -758,7 +754,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                     const int valid = min(kKeys, x.kv_limit - base);
                     const int nc = (valid + kChunk - 1) / kChunk;
                     const bool tail = valid < kKeys;
-                    const uint32_t full = map_to(bar_vfull(st), 0);
+                    const uint32_t full = map_to(bar_kvfull(st), 0);
                     if (lane == 0) {
                         if (tail) mbar_expect_tx(bar_vtail, (uint32_t)(nc * kChunk * 128));
                         else mbar_expect_tx_cluster(full, (uint32_t)(nc * kChunk * 128));
@@ -799,7 +795,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         if (tail_pending) drain_phase(bar_vtail, tails & 1);
         if (rank == 0) {
             for (int i = max(0, issued - stages); i < issued; ++i)
-                drain_phase(is_k ? bar_kfull(i % stages) : bar_vfull(i % stages), (i / stages) & 1);
+                drain_phase(bar_kvfull(i % stages), (i / stages) & 1);
             if (is_k)
                 for (int ui = max(0, units_q - 2); ui < units_q; ++ui) drain_phase(bar_q(ui & 1), (ui >> 1) & 1);
         }
@@ -819,19 +815,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                 if (!warp_wait(bar_q(qb), (ui >> 1) & 1, abort, p.status)) { ok = false; break; }
                 const uint64_t dq = dQ + (uint64_t)((qb * kQBytes) >> 4);
                 // A barrier poll costs a shared-memory round trip while the tensor
-                // core streams operands: the next group's K or V barrier is tested
+                // core streams operands: the next tile's K/V barrier is tested
                 // before the current group's MMAs are issued (the result is used
                 // after them), and waited for only if it had not completed.
                 bool k_seen = false;
                 for (int n = 0; ok && n <= x.ntiles; ++n) {
-                    bool v_seen = false;
                     if (n < x.ntiles) {
-                        const int t = t0 + n, st = t % kKStages, b = t & 1;
-                        if (!__all_sync(0xffffffffu, k_seen) && !warp_wait(bar_kfull(st), (t / kKStages) & 1, abort, p.status)) { ok = false; break; }
-                        if (n >= 1) {
-                            const int tv = t - 1;
-                            v_seen = mbar_test(bar_vfull(tv % kVStages), (tv / kVStages) & 1);
-                        }
+                        const int t = t0 + n, st = t % kStages, b = t & 1;
+                        if (!__all_sync(0xffffffffu, k_seen) && !warp_wait(bar_kvfull(st), (t / kStages) & 1, abort, p.status)) { ok = false; break; }
                         tc_fence_after();
                         if (lane == 0) {
                             const uint64_t kd = dK + (uint64_t)((st * kKStage) >> 4);
@@ -841,15 +832,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                                       kd + (uint64_t)(((kk >> 2) * kKHalf + (kk & 3) * 32) >> 4), idS, kk > 0);
                             }
                             umma_commit_pair(bar_sfull(b));
-                            umma_commit_pair(bar_kfree(st));
                             if (n == x.ntiles - 1) umma_commit_pair(bar_qfree(qb));  // Q buffer qb is free again
                         }
                         __syncwarp();
                     }
                     k_seen = false;
                     if (n >= 1) {
-                        const int m = n - 1, t = t0 + m, st = t % kVStages;
-                        if (!__all_sync(0xffffffffu, v_seen) && !warp_wait(bar_vfull(st), (t / kVStages) & 1, abort, p.status)) { ok = false; break; }
+                        const int m = n - 1, t = t0 + m, st = t % kStages;
                         if (!warp_wait(bar_pfull(t & 1), (t >> 1) & 1, abort, p.status)) { ok = false; break; }
                         // The unit's first P V into each O buffer overwrites it: the
                         // previous unit's O_0 and O_1 must have been read out by both
@@ -857,7 +846,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                         if (m == 0 && ui > 0 && !warp_wait(bar_ofree, (ui - 1) & 1, abort, p.status)) { ok = false; break; }
                         if (n + 1 < x.ntiles) {
                             const int tk = t0 + n + 1;
-                            k_seen = mbar_test(bar_kfull(tk % kKStages), (tk / kKStages) & 1);
+                            k_seen = mbar_test(bar_kvfull(tk % kStages), (tk / kStages) & 1);
                         }
                         tc_fence_after();
                         if (lane == 0) {
@@ -867,8 +856,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                             for (int kk = 0; kk < kKeys / 16; ++kk)
                                 umma2_ts(tmem + kColO + (t & 1) * kD, pt + kk * 8, vd + (uint64_t)((kk * (16 * 128)) >> 4), idO,
                                          (m > 1 || kk > 0) ? 1u : 0u);
-                            umma_commit_pair(bar_pfree(t & 1));
-                            umma_commit_pair(bar_vfree(st));
+                            umma_commit_pair(bar_kvfree(st));  // this tile's P V done: its K and V stages are free
                         }
                         __syncwarp();
                     }
@@ -931,7 +919,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                 const float alpha = grow ? ex2(m_ref - m_tile) : 1.f;
                 if (n >= 2 && __any_sync(0xffffffffu, grow)) {
                     // O_G must hold this group's earlier tiles before it is rescaled.
-                    if (!warp_wait_sleep(bar_pfree(G), ((t - 2) >> 1) & 1, abort, p.status)) { ok = false; break; }
+                    if (!warp_wait_sleep(bar_kvfree((t - 2) % kStages), ((t - 2) / kStages) & 1, abort, p.status)) { ok = false; break; }
                     tc_fence_after();
 #pragma unroll
                     for (int c = 0; c < 4; ++c) {
@@ -992,7 +980,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                 // wait cannot pass on an older phase.
                 if (!warp_wait_sleep(bar_xfull(quarter), ui & 1, abort, p.status)) { ok = false; break; }
                 const int tl_last = t0 + x.ntiles - 1;
-                if (!warp_wait_sleep(bar_pfree(tl_last & 1), (tl_last >> 1) & 1, abort, p.status)) { ok = false; break; }
+                if (!warp_wait_sleep(bar_kvfree(tl_last % kStages), (tl_last / kStages) & 1, abort, p.status)) { ok = false; break; }
                 const float2 o1 = xs[r];
                 __syncwarp();
                 if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar_xempty(quarter)) : "memory");
