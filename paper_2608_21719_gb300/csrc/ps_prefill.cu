@@ -53,10 +53,12 @@
 // O_1 at 256 and 384), so that one group computes while the other waits for
 // its next score tile and the tensor core works on both: two softmax streams
 // per SM sub-partition where one left the sub-partition idle during every
-// wait.  At the end of a unit group 1 hands (m, l) of each row to group 0
-// through shared memory and group 0 merges the halves -- O = (2^(m_0 - m) O_0
-// + 2^(m_1 - m) O_1) / (2^(m_0 - m) l_0 + 2^(m_1 - m) l_1), m = max(m_0, m_1)
-// -- and writes the row.  P over S needs no barrier of its own: the Q K^T of
+// wait.  At the end of a unit the group that did not run its last tile hands
+// (m, l) of each row through shared memory to the group that did, which
+// merges the halves -- O = (2^(m_0 - m) O_0 + 2^(m_1 - m) O_1) / (2^(m_0 - m)
+// l_0 + 2^(m_1 - m) l_1), m = max(m_0, m_1) -- and writes the row, while the
+// handing group (which owns the next unit's first tile) runs that tile's
+// softmax.  P over S needs no barrier of its own: the Q K^T of
 // tile n + 2 is issued after the P V of tile n, and tcgen05 MMAs of one
 // thread run in order.  The softmax's instruction stream is what the MMA
 // issue competes with on every SM sub-partition, so it is kept short: a
@@ -74,8 +76,8 @@
 // work (descending, in a snake over the clusters), with the rings, the S/P
 // buffers and their barrier phases running on from one unit to the next: the
 // next unit's Q (double-buffered) and first K/V tiles load while the current
-// unit finishes, and its first Q K^T runs while softmax group 0 merges and
-// writes out the current unit's rows.  (Batches with more units than fit a cluster's list run
+// unit finishes, and its first Q K^T and softmax run while the other group
+// merges and writes out the current unit's rows.  (Batches with more units than fit a cluster's list run
 // one unit per cluster.)
 //
 // Every mbarrier wait gives up after ~2 s of globaltimer, or at once when
@@ -647,7 +649,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     volatile int *abort = reinterpret_cast<volatile int *>(bars + kB + 7);
     auto bar_qfree = [&](int qb) { return saddr(bars + kB + 8 + qb); };  // [2]
     const uint32_t bar_ofree = saddr(bars + kB + 10);                    // leader's
-    auto bar_xfull = [&](int q) { return saddr(bars + kB + 11 + q); };   // [4] group 1 -> group 0, per lane quarter
+    auto bar_xfull = [&](int q) { return saddr(bars + kB + 11 + q); };   // [4] (m, l) hand-off to the merging group, per lane quarter
     auto bar_xempty = [&](int q) { return saddr(bars + kB + 15 + q); };  // [4]
     const uint32_t bar_stall = saddr(bars + kB + 19);  // nothing arrives on it: the injected stall (tests only)
     static_assert((2 + 2 * kStages + 20) * 8 <= kBarBytes, "barrier area");
@@ -667,7 +669,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         }
         mbar_init(bar_mma_end, 1);
         mbar_init(bar_vtail, 1);
-        mbar_init(bar_ofree, 8);  // both CTAs' group 0 softmax warps have read O
+        mbar_init(bar_ofree, 8);  // both CTAs' merging softmax warps have read O
         mbar_init(bar_stall, 1);
         for (int q = 0; q < 4; ++q) {
             mbar_init(bar_xfull(q), 1);
@@ -842,7 +844,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                         if (!warp_wait(bar_pfull(t & 1), (t >> 1) & 1, abort, p.status)) { ok = false; break; }
                         // The unit's first P V into each O buffer overwrites it: the
                         // previous unit's O_0 and O_1 must have been read out by both
-                        // CTAs' group 0 softmax warps (the merge).
+                        // CTAs' merging softmax warps.
                         if (m == 0 && ui > 0 && !warp_wait(bar_ofree, (ui - 1) & 1, abort, p.status)) { ok = false; break; }
                         if (n + 1 < x.ntiles) {
                             const int tk = t0 + n + 1;
@@ -968,31 +970,35 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             if (!ok) break;
             float la, lb;
             unpack2(l2, la, lb);
-            if (G == 1) {
-                // Hand (m, l) of these rows to group 0, which merges the two halves.
+            // The group of the unit's last tile merges: the other group finished
+            // its last tile a tile earlier and owns the next unit's first tile,
+            // whose softmax then runs alongside the merge.
+            const int tl_last = t0 + x.ntiles - 1;
+            if (G != (tl_last & 1)) {
+                // Hand (m, l) of these rows to the merging group.
                 if (ui > 0 && !warp_wait_sleep(bar_xempty(quarter), (ui - 1) & 1, abort, p.status)) { ok = false; break; }
                 xs[r] = make_float2(m_ref, la + lb);
                 __syncwarp();
                 if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar_xfull(quarter)) : "memory");
             } else {
-                // Group 1's hand-off comes after its last softmax, so the barrier of
-                // the unit's last P V is then at most one phase behind: its parity
-                // wait cannot pass on an older phase.
+                // This group's S-full wait of tile tl_last implies the P V of tile
+                // tl_last - 2, so the barrier of the unit's last P V is at most one
+                // phase behind: its parity wait cannot pass on an older phase.
                 if (!warp_wait_sleep(bar_xfull(quarter), ui & 1, abort, p.status)) { ok = false; break; }
-                const int tl_last = t0 + x.ntiles - 1;
                 if (!warp_wait_sleep(bar_kvfree(tl_last % kStages), (tl_last / kStages) & 1, abort, p.status)) { ok = false; break; }
                 const float2 o1 = xs[r];
                 __syncwarp();
                 if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar_xempty(quarter)) : "memory");
-                // Which buffers this unit's tiles used (a one-tile unit uses one).
-                const bool has0 = x.ntiles >= 2 || (t0 & 1) == 0, has1 = x.ntiles >= 2 || (t0 & 1) == 1;
+                // The other group has tiles in this unit unless it has one tile
+                // (which is this group's).
+                const bool has1 = x.ntiles >= 2;
                 const float m0 = m_ref, m1 = o1.x;
-                const float m = fmaxf(has0 ? m0 : -INFINITY, has1 ? m1 : -INFINITY);
-                const float c0 = has0 ? ex2(m0 - m) : 0.f, c1 = has1 ? ex2(m1 - m) : 0.f;
+                const float m = fmaxf(m0, has1 ? m1 : -INFINITY);
+                const float c0 = ex2(m0 - m), c1 = has1 ? ex2(m1 - m) : 0.f;
                 const float inv = 1.f / ((la + lb) * c0 + o1.y * c1);
                 const float f0 = c0 * inv, f1 = c1 * inv;
                 tc_fence_after();
-                // O = f0 O_0 + f1 O_1, 32 dims at a time, straight to the output
+                // O = f0 O_G + f1 O_{1-G}, 32 dims at a time, straight to the output
                 // row; then the leader may start the next unit's P V (which
                 // overwrites both accumulators).
                 uint16_t *orow = row_valid ? p.out + ((size_t)(x.qs0 + tok0 + tl) * p.num_q_heads + (size_t)x.j * g + hl) * kD : nullptr;
@@ -1001,15 +1007,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                     // Both accumulators are read; one this unit left unused holds
                     // stale values and is not used.
                     float a0[32], a1[32];
-                    tmem_ld32(trow + kColO + c * 32, a0);
-                    tmem_ld32(trow + kColO + kD + c * 32, a1);
+                    tmem_ld32(trow + kColO + G * kD + c * 32, a0);
+                    tmem_ld32(trow + kColO + (G ^ 1) * kD + c * 32, a1);
                     tmem_wait_ld();
                     tmem_loaded<32>(a0);
                     tmem_loaded<32>(a1);
                     uint32_t w[16];
 #pragma unroll
                     for (int e = 0; e < 16; ++e) {
-                        float y0 = has0 ? a0[2 * e] * f0 : 0.f, y1 = has0 ? a0[2 * e + 1] * f0 : 0.f;
+                        float y0 = a0[2 * e] * f0, y1 = a0[2 * e + 1] * f0;
                         y0 = has1 ? fmaf(a1[2 * e], f1, y0) : y0;
                         y1 = has1 ? fmaf(a1[2 * e + 1], f1, y1) : y1;
                         const __nv_bfloat162 pr = __floats2bfloat162_rn(y0, y1);

@@ -3,7 +3,8 @@
 `ps_prefill.cu` runs one CTA pair per persistent cluster with these roles per
 CTA: a K producer (which also loads Q, double-buffered per unit), a V
 producer, the MMA issuer (leader CTA only), and two softmax groups (even and
-odd key tiles) of which group 0 merges the two halves at the end of a unit.
+odd key tiles); at the end of a unit the group that ran its last tile merges
+the two halves, after the other group has handed over its (m, l).
 Every wait is a parity wait on an mbarrier, which is sound only while the
 barrier has completed exactly the awaited phase's predecessor or the awaited
 phase itself: one phase further behind and the wait passes at once, one phase
@@ -47,7 +48,8 @@ class _Model:
         self.errors = []
         self.mma = []       # issued, not yet complete: ('op', key) or ('commit', barrier)
         self.finished = set()
-        self.o_read = set()  # (rank, unit): group 0 has read O_0 and O_1 of the unit
+        self.o_read = set()  # (rank, unit): the merging group has read O_0 and O_1 of the unit
+        self.xs = {}         # rank -> ('written', unit) or the last unit read
         self.last_qk = {}    # unit -> global index of its last tile
         b = {}
         for st in range(STAGES):
@@ -58,9 +60,9 @@ class _Model:
             b['qfree', i] = _Bar(1)
             b['sfull', i] = _Bar(1)
             b['pfull', i] = _Bar(8)    # the group's four warps in each CTA
-        b['ofree'] = _Bar(8)           # group 0's four warps in each CTA
+        b['ofree'] = _Bar(8)           # the merging group's four warps in each CTA
         for r in range(2):
-            b['xfull', r] = _Bar(1)    # per CTA: group 1 -> group 0 hand-off
+            b['xfull', r] = _Bar(1)    # per CTA: (m, l) hand-off to the merging group
             b['xempty', r] = _Bar(1)
         self.b = b
 
@@ -155,13 +157,17 @@ class _Model:
                     self.errors.append('P of tile %d written over S before the P V of tile %d' % (t, t - 2))
                 yield from self.pause(6)
                 self.b['pfull', G].arrive(4)
-            if G == 1:
+            last = t0 + nt - 1
+            merger = last & 1  # the group of the unit's last tile merges
+            if G != merger:
                 if ui > 0:
                     while not self.ready(('xempty', rank), ui - 1):
                         yield
+                if self.xs.get(rank, -1) != ui - 1:
+                    self.errors.append('hand-off of unit %d overwrites one not yet read' % ui)
+                self.xs[rank] = ('written', ui)
                 self.b['xfull', rank].arrive()
             else:
-                last = t0 + nt - 1
                 while not self.ready(('xfull', rank), ui):
                     yield
                 # After the hand-off group 1's last softmax has passed its S-full
@@ -172,6 +178,9 @@ class _Model:
                 missing = [t for t in range(t0, t0 + nt) if ('PV', t) not in self.finished]
                 if missing:
                     self.errors.append('O read out before the P V of tiles %s' % missing)
+                if self.xs.get(rank) != ('written', ui):
+                    self.errors.append('merge of unit %d read a hand-off that is not its own' % ui)
+                self.xs[rank] = ui
                 self.b['xempty', rank].arrive()
                 yield from self.pause(3)
                 self.o_read.add((rank, ui))
