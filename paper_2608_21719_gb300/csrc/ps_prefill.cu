@@ -129,7 +129,7 @@ constexpr int kOffBar = kOffV + kStages * kVStage;
 constexpr int kBarBytes = 512;
 constexpr int kMaxUnitsPerCluster = 256;            // a cluster's unit list (persistent mode)
 constexpr int kOffList = kOffBar + kBarBytes;
-constexpr int kOffX = kOffList + kMaxUnitsPerCluster * 4;  // (m, l) of group 1 rows for the merge
+constexpr int kOffX = kOffList + kMaxUnitsPerCluster * 4;  // (m, l) of the handing group's rows for the merge
 constexpr int kSmemBytes = 1024 + kOffX + kRows * 8;  // 1 KiB of alignment slack
 // Persistent mode needs the whole batch's units (sequence x KV head x pair of
 // query tiles) below this; the host launches one unit per cluster above it.
