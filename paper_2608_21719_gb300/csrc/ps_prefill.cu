@@ -912,10 +912,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                     for (int i = 0; i < kKeys; ++i)
                         if (base + i >= limit) sv[i] = -INFINITY;
                 }
-                float mx = sv[0];
+                // Two independent max chains over the halves of the row.
+                float mxa = sv[0], mxb = sv[64];
 #pragma unroll
-                for (int i = 1; i + 1 < kKeys; i += 2) mx = max3(mx, sv[i], sv[i + 1]);
-                mx = fmaxf(mx, sv[kKeys - 1]);
+                for (int i = 1; i + 1 < 64; i += 2) {
+                    mxa = max3(mxa, sv[i], sv[i + 1]);
+                    mxb = max3(mxb, sv[64 + i], sv[64 + i + 1]);
+                }
+                float mx = max3(mxa, mxb, fmaxf(sv[63], sv[127]));
                 const float m_tile = mx * sl2;
                 const bool grow = m_tile > m_ref + kRescaleLog2;
                 const float alpha = grow ? ex2(m_ref - m_tile) : 1.f;
