@@ -255,7 +255,9 @@ ps_status_t ps_kv_unpack(const void *src, const long long *src_offsets, const in
  *   max_q_len    an upper bound on Q_s over the batch (sizes the grid; the
  *                query tiles past a sequence's Q_s do nothing; a chunk longer
  *                than max_q_len has its rows past it left unwritten and raises
- *                PS_DEVICE_LEN_CLAMPED)
+ *                PS_DEVICE_LEN_CLAMPED).  With max_q_len, num_seqs or
+ *                total_q_tokens 0 the call launches nothing and returns PS_OK
+ *                (no row is written and no flag raised).
  *   device_status  optional device word that receives PS_DEVICE_* flags
  * A sequence with Q_s > seq_lens[s], a negative Q_s, a length above
  * max_blocks_per_seq * block_size or rows outside [0, total_q_tokens) is

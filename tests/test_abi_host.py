@@ -225,3 +225,42 @@ def test_fault_injection_arguments():
     psd.ps_test_inject(psd.PS_INJECT_DECODE_STALL, 0)
     psd.ps_test_inject(psd.PS_INJECT_PREFILL_STALL, 10**6)
     psd.ps_test_inject(psd.PS_INJECT_PREFILL_STALL, 0)
+
+
+def test_prefill_validates_on_the_host():
+    # Stand-in 16-byte-aligned device addresses: every case below is decided
+    # before the call encodes a tensor map or touches the device.
+    A = 256
+    base = [A, A, A, A, A, A, A, 1, 5, 5, 8, 2, 128, 16, 4, 16, 0.1, None, None]
+
+    def status(**changes):
+        args = list(base)
+        names = ["q", "k", "v", "bt", "sl", "qs", "out", "num_seqs", "total", "max_q", "hq", "hkv", "hd", "bs",
+                 "mbps", "nb", "scale", "dev_status", "stream"]
+        for k, v in changes.items():
+            args[names.index(k)] = v
+        try:
+            psd.ps_prefill_attention(*args)
+        except psd.PsError as e:
+            return e.status
+        return psd.PS_OK
+
+    inval, unsup = psd.PS_ERR_INVALID_ARG, psd.PS_ERR_UNSUPPORTED
+    assert status(q=0) == inval
+    assert status(out=A + 8) == inval            # bf16 rows need 16-byte alignment
+    assert status(bt=A + 2) == inval             # int32 arrays need 4-byte alignment
+    assert status(dev_status=A + 1) == inval
+    assert status(num_seqs=-1) == inval
+    assert status(max_q=6) == inval              # above total_q_tokens
+    assert status(hq=8, hkv=3) == inval          # heads not a multiple
+    assert status(nb=0) == inval
+    assert status(scale=float("inf")) == inval
+    assert status(hd=64) == unsup
+    assert status(hq=34, hkv=2) == unsup         # g = 17
+    assert status(bs=8) == unsup                 # not a multiple of 16
+    assert status(num_seqs=65536) == unsup
+    assert status(total=10 ** 7, max_q=10 ** 7, hq=2, hkv=2) == unsup  # more than 65535 query tiles
+    # nothing to do: no launch, no device call, PS_OK
+    assert status(num_seqs=0) == psd.PS_OK
+    assert status(total=0, max_q=0) == psd.PS_OK
+    assert status(max_q=0) == psd.PS_OK
