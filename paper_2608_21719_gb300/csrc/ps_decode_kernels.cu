@@ -1013,9 +1013,11 @@ __global__ void __launch_bounds__(kWorkersPerCta * 32, 1)
 cudaError_t launch_decode(const DecodeParams &p, const CUtensorMap &tmK, const CUtensorMap &tmV, int grid_ctas,
                           size_t smem_bytes, cudaStream_t stream) {
     // Allow the kernel the largest dynamic shared memory the device offers
-    // (its opt-in limit less the kernel's static shared memory), once per
-    // device.  Every caller sets the same value, so concurrent first launches
-    // on one device cannot leave a smaller limit behind.
+    // (its opt-in limit less the kernel's static shared memory).  The limit is
+    // a property of the device and this binary and is computed once; the
+    // attribute belongs to the current context and is set on every call, so
+    // a context created after cudaDeviceReset() gets it too.  Every caller
+    // sets the same value, so concurrent calls cannot leave a smaller one.
     static std::atomic<int> attr_limit[64];
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
@@ -1029,12 +1031,12 @@ cudaError_t launch_decode(const DecodeParams &p, const CUtensorMap &tmK, const C
             (e = cudaFuncGetAttributes(&fa, ps_decode_kernel)) != cudaSuccess)
             return e;
         limit = optin - (int)fa.sharedSizeBytes;
-        if ((e = cudaFuncSetAttribute(ps_decode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, limit)) !=
-            cudaSuccess)
-            return e;
         attr_limit[dev].store(limit, std::memory_order_release);
     }
     if (smem_bytes > (size_t)limit) return cudaErrorInvalidValue;
+    if ((e = cudaFuncSetAttribute(ps_decode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, limit)) !=
+        cudaSuccess)
+        return e;
     if ((e = take_injected_launch_error()) != cudaSuccess) return e;
     DecodeParams q = p;
     q.test_stall_ns = take_injected_stall_ns();
